@@ -1,0 +1,267 @@
+/*
+ * lsp.h -- C ABI of the fixed-cost drafting round (LongSpark, arxiv 2609.37029).
+ *
+ * One drafting round (Sec. 2.4 "Inference", Fig. 2):
+ *   1. lsp_view_update: fold the target verification pass's newly accepted rows
+ *      into the fixed-size context interface -- the global summary (Eq.
+ *      global-summary maintained by the merge of App. A.2, Eq. summary-update),
+ *      the recent KV window and the boundary hidden states (Sec. 2.2).
+ *   2. lsp_draft: the block-diffusion drafter forward over [block; window;
+ *      summary] (Sec. 2.3, Eq. draft-context, App. A.1), the frozen final norm
+ *      and LM head (base logits z^(0)), then lsp_sample's correction+sampling.
+ *   3. lsp_sample: the low-rank Markov correction (Eq. markov) and sequential
+ *      sampling of the B proposals (Eq. proposal-factorization).
+ *
+ * Conventions shared by every call:
+ *   - Every call returns an int status: LSP_OK (0) or a negative LSP_ERR_*.
+ *     Argument and shape errors are detected on the host before any launch and
+ *     nothing is enqueued then.  No exception or abort crosses the ABI.
+ *   - All device work is enqueued on the caller's stream (lsp_stream_t is a
+ *     cudaStream_t; NULL means the legacy default stream) and returns without
+ *     synchronising, except where a call says otherwise.
+ *   - Pointers documented as "device" must be device (or managed) memory owned
+ *     by the caller, valid until the enqueued work completes.  The library owns
+ *     only what lsp_state_create allocates.
+ *   - Element type of every tensor argument documented as "dtype" is the
+ *     config's dtype: LSP_DTYPE_BF16 (bfloat16) or LSP_DTYPE_F32 (float).
+ *   - Errors a kernel detects (a token id out of range, accepted_len beyond the
+ *     row capacity, a bounded wait that timed out) set bits of a device error
+ *     word (LSP_DEV_*) read by lsp_get_error; kernels never trap.
+ *   - Layouts are dense and row-major; linear weights are [out][in] with `in`
+ *     contiguous (y = W x).
+ */
+#ifndef LSP_H
+#define LSP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LSP_MAX_DRAFT_LAYERS 16
+
+/* status codes */
+#define LSP_OK 0
+#define LSP_ERR_ARG (-1)          /* null pointer / invalid scalar argument */
+#define LSP_ERR_SHAPE (-2)        /* config or size outside what the kernels support */
+#define LSP_ERR_CUDA (-3)         /* a CUDA runtime or driver call failed */
+#define LSP_ERR_TIMEOUT (-4)      /* a device wait gave up (see lsp_get_error) */
+#define LSP_ERR_STATE (-5)        /* state not initialised or device error pending */
+#define LSP_ERR_NOMEM (-6)        /* device allocation failed in lsp_state_create */
+#define LSP_ERR_UNSUPPORTED (-7)  /* no sm_103a device / feature unavailable */
+
+/* device error word bits (lsp_get_error) */
+#define LSP_DEV_TIMEOUT 1u        /* a bounded mbarrier/flag wait expired */
+#define LSP_DEV_BAD_TOKEN 2u      /* a token id outside [-1, V) (slot 0: outside [0, V)) */
+#define LSP_DEV_BAD_DELTA 4u      /* accepted_len outside [0, row capacity] */
+
+#define LSP_DTYPE_BF16 0
+#define LSP_DTYPE_F32 1
+
+typedef void* lsp_stream_t;       /* cudaStream_t */
+typedef struct lsp_state lsp_state; /* opaque, library-owned */
+
+/*
+ * Shapes of one drafter + target pairing.
+ *   C   concurrency: requests processed together (state rows)
+ *   B   draft block slots = proposals per round (Sec. 2.3)
+ *   L   tapped target layers (the set of Sec. 2.2; App. B.1 uses 5)
+ *   D   drafter layers (App. B.1: 5)
+ *   H   hidden size; nq / nkv query / key-value heads of head dim d (the
+ *       target's, since draft queries score target window keys)
+ *   F   drafter MLP width; V vocabulary; rc rank of the Markov correction
+ *   W   recent window rows per tapped layer (App. B.1: 256)
+ *   R   summary queries per tapped layer and query head (App. B.1: 16)
+ *   layer_map[j]  tapped-layer index draft layer j reads its window and summary
+ *       from (Sec. 2.3 pairs draft layer j with tapped layer l(j)); a value < 0
+ *       selects floor(j * L / D)
+ *   rope_theta  rotary base of the drafter's block queries/keys; rms_eps RMSNorm eps
+ * Supported: dtype BF16 with d == 128, B <= 16, nq % nkv == 0, nq/nkv <= 8;
+ * dtype F32 with d <= 128 even; H, nq*d, nkv*d, F multiples of 64; C*B <= 512.
+ */
+typedef struct lsp_config {
+  int C, B, L, D, H, nq, nkv, d, F, V, W, R, rc;
+  int dtype;
+  int layer_map[LSP_MAX_DRAFT_LAYERS];
+  float rope_theta;
+  float rms_eps;
+} lsp_config;
+
+/*
+ * New target rows of one verification pass (Sec. 2.1, 2.4): for request b,
+ * tapped layer l and new row j < accepted_len[b]:
+ *   k[b][l][j][0..nkv)[0..d)   key rows as cached by the target (rotary applied)
+ *   v[b][l][j][0..nkv)[0..d)   value rows
+ *   h[b][l][j][0..H)           hidden state at that row (only row accepted_len-1 is read)
+ * All three are device pointers of dtype with row capacity `rows` per (b, l).
+ */
+typedef struct lsp_target_feats {
+  const void* k;
+  const void* v;
+  const void* h;
+  int rows;
+} lsp_target_feats;
+
+/* One Qwen3-style draft layer (App. B.1); device pointers of dtype. */
+typedef struct lsp_layer_weights {
+  const void* in_norm;    /* [H] */
+  const void* wq;         /* [nq*d][H] */
+  const void* wk;         /* [nkv*d][H] */
+  const void* wv;         /* [nkv*d][H] */
+  const void* q_norm;     /* [d] per-head RMSNorm of block queries */
+  const void* k_norm;     /* [d] per-head RMSNorm of block keys */
+  const void* wo;         /* [H][nq*d] */
+  const void* post_norm;  /* [H] */
+  const void* w_gate;     /* [F][H] */
+  const void* w_up;       /* [F][H] */
+  const void* w_down;     /* [H][F] */
+} lsp_layer_weights;
+
+/* Drafter weights (device pointers of dtype). The target's embedding, final
+ * norm and LM head are reused frozen (Sec. 2.3, App. B.1). */
+typedef struct lsp_weights {
+  const void* embed;       /* [V][H] target token embedding */
+  const void* final_norm;  /* [H] target final RMSNorm weight */
+  const void* lm_head;     /* [V][H] target vocabulary head */
+  const void* fuse;        /* [H][L*H] boundary fusion: c_t = fuse . [h^l1;...;h^lL] (Sec. 2.2) */
+  const void* pos;         /* [B][H] within-block positional encodings (Sec. 2.3) */
+  const void* mask_emb;    /* [H] mask-token embedding of slots 1..B-1 */
+  const void* Ec;          /* [V][rc] correction embedding E_c (Eq. markov) */
+  const void* Wc;          /* [V][rc] correction output map W_c (Eq. markov) */
+  lsp_layer_weights layer[LSP_MAX_DRAFT_LAYERS];
+} lsp_weights;
+
+/*
+ * Sampling of the proposals (Eq. proposal-factorization).  temperature == 0:
+ * greedy, y_i = argmax_v z_i[v].  temperature > 0: Gumbel-max,
+ * y_i = argmax_v (z_i[v] / T + g), g = -log(-log u), u = ((x >> 9) + 0.5) * 2^-23,
+ * x = word (v & 3) of Philox4x32-10 with key (seed lo32, seed hi32) and counter
+ * (v >> 2, i, b, round).  Ties go to the lowest vocabulary index.
+ */
+typedef struct lsp_sample_params {
+  float temperature;
+  uint32_t round;
+  uint64_t seed;
+} lsp_sample_params;
+
+/* Human-readable name of a status code (static string). */
+const char* lsp_status_string(int status);
+
+/* Bytes of the persistent per-state interface for `cfg` (window, summary
+ * (m, eta), boundary h, counters), all C requests: a function of the shapes
+ * only, never of the prefix length (Sec. 2.4 "Fixed-cost complexity").
+ * Returns 0 for an invalid config. Host-only; needs no GPU. */
+size_t lsp_state_bytes(const lsp_config* cfg);
+
+/* Validate `cfg` on the host. LSP_OK or LSP_ERR_SHAPE / LSP_ERR_ARG. Needs no GPU. */
+int lsp_config_check(const lsp_config* cfg);
+
+/* Allocate a state on the current device: the interface (lsp_state_bytes) and
+ * a fixed workspace for the drafter's activations, logits and sampler
+ * partials.  Synchronous; the only call that allocates device memory.  The
+ * state starts uninitialised (call lsp_state_init). */
+int lsp_state_create(const lsp_config* cfg, lsp_state** out);
+
+/* Free everything lsp_state_create allocated (synchronises the device first).
+ * NULL is ignored. */
+void lsp_state_destroy(lsp_state* st);
+
+/* Reset the interface to the empty prefix -- m = 0, eta = -inf, empty window,
+ * zero boundary, t = 0, device error word cleared -- and copy the summary
+ * queries G (device, dtype, [L][nq][R][d]; Sec. 2.2, App. B.2 "Summary
+ * queries", held fixed during inference) into the state.  The summary over a
+ * prefix is then built by lsp_view_update calls over its rows in chunks of any
+ * size (the merge of App. A.2 makes the chunking exact); this is the one-time
+ * O(t) prefill the paper attributes to target prefill (Fig. 3). */
+int lsp_state_init(lsp_state* st, const void* G, lsp_stream_t stream);
+
+/* Fold accepted_len[b] new target rows of request b (device int32 [C], each in
+ * [0, feats->rows]; 0 leaves request b untouched) into the interface:
+ *  - summary: for every tapped layer l, query head h and summary query r,
+ *    the attention statistics of g_r over the new keys of KV head h/(nq/nkv)
+ *    are merged into (eta, m) by Eq. summary-update;
+ *  - window: the new K/V rows enter the ring of the last W rows (row p of the
+ *    prefix lives in slot p mod W);
+ *  - boundary: h of the last new row replaces the boundary state;
+ *  - t += accepted_len[b].
+ * Reads only the new rows, never the prefix (Sec. 2.4). */
+int lsp_view_update(lsp_state* st, const lsp_target_feats* feats,
+                    const int32_t* accepted_len, lsp_stream_t stream);
+
+/* One drafter forward for all C requests (Sec. 2.3, App. A.1) followed by the
+ * sampler of lsp_sample.
+ *   block_tokens  device int32 [C][B]: slot 0 = committed token a (also y_0 of
+ *                 the Markov correction); slots >= 1: -1 for the mask embedding
+ *                 or a token id to embed
+ *   w             weights (host struct of device pointers)
+ *   sp            sampling parameters (host struct)
+ *   out_tokens    device int32 [C][B]: proposals y_1..y_B
+ *   out_logits    device float [C][B][V] corrected logits z_i (the verification
+ *                 distributions q_i = softmax(z_i)), or NULL to skip writing them
+ * Rotary positions of slot i are t + i (t = rows folded so far).  Uses only
+ * the state's fixed workspace; allocates nothing. */
+int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
+              const lsp_sample_params* sp, int32_t* out_tokens, float* out_logits,
+              lsp_stream_t stream);
+
+/* Correction + sampling alone (Eq. markov, Eq. proposal-factorization) on given
+ * base logits, with the state's config (C, B, V, rc, dtype) and workspace:
+ *   base_logits  device float [C][B][V] (z^(0); not modified)
+ *   prev_token   device int32 [C]: y_0 = a of each request
+ *   Ec, Wc       device dtype [V][rc]
+ *   out_tokens   device int32 [C][B]; out_logits device float [C][B][V] or NULL
+ * For i = 1..B in order: z_i = z_i^(0) + W_c E_c[y_{i-1}], y_i drawn per sp. */
+int lsp_sample(lsp_state* st, const float* base_logits, const int32_t* prev_token,
+               const void* Ec, const void* Wc, const lsp_sample_params* sp,
+               int32_t* out_tokens, float* out_logits, lsp_stream_t stream);
+
+/* Dense projection Y = X W^T with the drafter's tensor-core GEMM (the kernel
+ * every projection of lsp_draft uses), for checking it on its own.
+ *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].
+ *   M <= 512, K and N multiples of 16 bytes / element size.
+ *   splits: split-K factor (1..16); workspace device bytes of at least
+ *   lsp_linear_workspace_bytes(M, N, splits), zero-filled before its first use
+ *   (the kernel leaves it reusable). */
+size_t lsp_linear_workspace_bytes(int M, int N, int splits);
+int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype,
+               int splits, void* workspace, size_t workspace_bytes, lsp_stream_t stream);
+
+/* Raw Philox4x32-10 words of the sampler stream, for checking the generator:
+ * out[n] (device uint32) = word (v & 3) of block (v >> 2) with v = n, counter
+ * (v >> 2, i, b, round) and key (seed lo32, seed hi32); n < count. */
+int lsp_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i,
+                     uint32_t* out, int count, lsp_stream_t stream);
+
+/* Stage timing hook (observability; no effect on results).  With n_events > 0,
+ * lsp_view_update and lsp_draft record the caller's CUDA events (cudaEvent_t
+ * handles, created by the caller with timing enabled, owned by the caller) at
+ * stage boundaries on the call's stream: stage k runs between events[k] and
+ * events[k+1].  Stages of one round, in order (lsp_stage_count / lsp_stage_name):
+ *   0 view_update, 1 fuse, 2 combine, then per draft layer j: qkv, attention,
+ *   o_proj, post_norm, gate_up, down, next_norm, then lm_head and sampler.
+ * n_events must be 0 (off) or lsp_stage_count(st) + 1.  Event records are
+ * capturable, so a captured round carries them as graph nodes. */
+int lsp_stage_count(lsp_state* st);
+const char* lsp_stage_name(lsp_state* st, int k);
+int lsp_set_stage_events(lsp_state* st, void* const* events, int n_events);
+
+/* Read (and clear, if clear != 0) the state's device error word into
+ * *dev_error (LSP_DEV_* bits).  Synchronises `stream`.  Returns LSP_OK,
+ * or LSP_ERR_TIMEOUT / LSP_ERR_STATE when bits are set. */
+int lsp_get_error(lsp_state* st, uint32_t* dev_error, int clear, lsp_stream_t stream);
+
+/* Copy the interface (exactly lsp_state_bytes(cfg) bytes, including t) to /
+ * from a host buffer, so a state can be checkpointed or built elsewhere.
+ * Synchronous on `stream`. Layout (all per state, dense, in this order):
+ *   win_k dtype [C][L][nkv][W][d], win_v dtype [C][L][nkv][W][d],
+ *   m float [C][L][nq][R][d], eta float [C][L][nq][R], h dtype [C][L][H],
+ *   t int64 [C]. */
+int lsp_state_export(lsp_state* st, void* host_buf, size_t bytes, lsp_stream_t stream);
+int lsp_state_import(lsp_state* st, const void* host_buf, size_t bytes, lsp_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LSP_H */

@@ -1,0 +1,437 @@
+// Fixed-context block attention of a draft layer (Sec. 2.3, Eq. draft-context).
+//
+// Each block query of request b and query head h attends, with one softmax
+// (scale 1/sqrt(d)) and no mask inside the block, over
+//     K = [K^b ; K^w ; G_h],   V = [V^b ; V^w ; M_h]
+// -- the B block keys/values of its KV head g = h / (nq/nkv), the valid rows
+// of the recent window of the paired tapped layer, and the R summary entries
+// of head h.  At most B + W + R entries per head, independent of t (Sec. 2.4).
+// The block q and k get the per-head RMSNorm and the rotary embedding here,
+// fused into the load of the q/k/v projection output.
+//
+// attn_mma_kernel (bf16, d = 128): one CTA per (request, KV head) stages the
+// window once in shared memory for all nq/nkv query heads (HBM traffic = one
+// read of the window and summary); warps are (query head x key split); each
+// warp runs an online softmax over 16-key chunks with mma.sync m16n8k16
+// (bf16 in, fp32 accumulate), and the key splits merge through shared memory.
+// attn_simple_kernel (fp32 storage): plain FMA version, one CTA per
+// (request, query head), for the fp32 reference shape.
+#include "common.cuh"
+#include "lsp_internal.h"
+
+namespace lsp {
+
+constexpr int kHD = 128;         // head dim of the tensor-core path
+constexpr int kLd = kHD + 8;     // smem row stride (bf16): 272 B, conflict-free ldmatrix
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_all;" ::: "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t* r, const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t* r, const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9},"
+      " {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+struct AttnLayout {
+  int rep, ksplit, nwarps, rows_bw;
+  size_t off_q, off_kbw, off_vbw, off_ks, off_vs, bytes;
+};
+
+static AttnLayout attn_layout(int B, int W, int nq, int nkv, int ksplit) {
+  AttnLayout a;
+  a.rep = nq / nkv;
+  a.ksplit = ksplit;
+  a.nwarps = a.rep * ksplit;
+  a.rows_bw = (B + W + 15) / 16 * 16;
+  const size_t row = kLd * sizeof(bf16);
+  a.off_q = 0;
+  a.off_kbw = a.off_q + (size_t)a.rep * 16 * row;
+  a.off_vbw = a.off_kbw + (size_t)a.rows_bw * row;
+  a.off_ks = a.off_vbw + (size_t)a.rows_bw * row;
+  a.off_vs = a.off_ks + (size_t)a.rep * 16 * row;
+  a.bytes = a.off_vs + (size_t)a.rep * 16 * row;
+  return a;
+}
+static size_t attn_merge_bytes(int nwarps) { return (size_t)nwarps * (16 * kHD + 32) * sizeof(float); }
+
+__global__ void __launch_bounds__(512)
+    attn_mma_kernel(const AttnParams p, const int rep, const int ksplit, const int rows_bw) {
+  extern __shared__ __align__(16) uint8_t asmem[];
+  const size_t row = kLd;
+  bf16* sQ = reinterpret_cast<bf16*>(asmem);
+  bf16* sKbw = sQ + (size_t)rep * 16 * row;
+  bf16* sVbw = sKbw + (size_t)rows_bw * row;
+  bf16* sKs = sVbw + (size_t)rows_bw * row;
+  bf16* sVs = sKs + (size_t)rep * 16 * row;
+
+  const int nwarps = rep * ksplit;
+  const int nthr = nwarps * 32;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int b = blockIdx.x / p.nkv, g = blockIdx.x % p.nkv;
+  const int B = p.B, L = p.L, l = p.layer;
+  const long long t = p.t[b];
+  const int count = (int)(t < p.W ? t : p.W);
+  const int nbw = B + count;                       // valid block + window keys
+  const int nbw16 = (nbw + 15) / 16 * 16;
+
+  // ---- window rows (valid slots are 0..count-1) straight into smem
+  const bf16* wk = static_cast<const bf16*>(p.win_k) + ((size_t)(b * L + l) * p.nkv + g) * p.W * kHD;
+  const bf16* wv = static_cast<const bf16*>(p.win_v) + ((size_t)(b * L + l) * p.nkv + g) * p.W * kHD;
+  for (int idx = tid; idx < count * 16; idx += nthr) {
+    const int r = idx >> 4, c = (idx & 15) * 8;
+    cp_async16(sKbw + (size_t)(B + r) * row + c, wk + (size_t)r * kHD + c);
+    cp_async16(sVbw + (size_t)(B + r) * row + c, wv + (size_t)r * kHD + c);
+  }
+  // ---- summary keys G_h (bf16) and values M_h (fp32 -> bf16)
+  const bf16* Gp = static_cast<const bf16*>(p.G) + ((size_t)l * p.nq + (size_t)g * rep) * p.R * kHD;
+  const float* Mp = p.m + (((size_t)(b * L + l) * p.nq + (size_t)g * rep) * p.R) * kHD;
+  for (int idx = tid; idx < rep * 16 * 16; idx += nthr) {
+    const int hr = idx >> 4, c = (idx & 15) * 8;     // hr = hh * 16 + r
+    const int hh = hr >> 4, r = hr & 15;
+    bf16* dk = sKs + (size_t)hr * row + c;
+    bf16* dv = sVs + (size_t)hr * row + c;
+    if (r < p.R) {
+      cp_async16(dk, Gp + ((size_t)hh * p.R + r) * kHD + c);
+      const float4* src = reinterpret_cast<const float4*>(Mp + ((size_t)hh * p.R + r) * kHD + c);
+      const float4 x0 = src[0], x1 = src[1];
+      uint4 o;
+      o.x = pack_bf16(x0.x, x0.y);
+      o.y = pack_bf16(x0.z, x0.w);
+      o.z = pack_bf16(x1.x, x1.y);
+      o.w = pack_bf16(x1.z, x1.w);
+      *reinterpret_cast<uint4*>(dv) = o;
+    } else {
+      *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
+    }
+  }
+  // ---- zero the tail of the last block/window chunk, and the padded query rows
+  for (int idx = tid; idx < (nbw16 - nbw) * 16; idx += nthr) {
+    const int r = nbw + (idx >> 4), c = (idx & 15) * 8;
+    *reinterpret_cast<uint4*>(sKbw + (size_t)r * row + c) = make_uint4(0, 0, 0, 0);
+    *reinterpret_cast<uint4*>(sVbw + (size_t)r * row + c) = make_uint4(0, 0, 0, 0);
+  }
+  for (int idx = tid; idx < rep * (16 - B) * 16; idx += nthr) {
+    const int hr = idx >> 4, c = (idx & 15) * 8;
+    const int hh = hr / (16 - B), i = B + hr % (16 - B);
+    *reinterpret_cast<uint4*>(sQ + (size_t)(hh * 16 + i) * row + c) = make_uint4(0, 0, 0, 0);
+  }
+  // ---- block q (rep heads), k, v of KV head g: per-head RMSNorm + rotary for q, k
+  {
+    const bf16* qkv = static_cast<const bf16*>(p.qkv);
+    const int ldq = (p.nq + 2 * p.nkv) * kHD;
+    const bf16* qn = static_cast<const bf16*>(p.q_norm);
+    const bf16* kn = static_cast<const bf16*>(p.k_norm);
+    const int kinds = rep + 2;
+    for (int item = warp; item < B * kinds; item += nwarps) {
+      const int i = item / kinds, kind = item % kinds;
+      const size_t mrow = (size_t)(b * B + i) * ldq;
+      const bf16* src;
+      bf16* dst;
+      if (kind < rep) {
+        src = qkv + mrow + (size_t)(g * rep + kind) * kHD;
+        dst = sQ + (size_t)(kind * 16 + i) * row;
+      } else if (kind == rep) {
+        src = qkv + mrow + (size_t)(p.nq + g) * kHD;
+        dst = sKbw + (size_t)i * row;
+      } else {
+        src = qkv + mrow + (size_t)(p.nq + p.nkv + g) * kHD;
+        dst = sVbw + (size_t)i * row;
+      }
+      float x[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) x[e] = to_f(src[lane + 32 * e]);
+      if (kind <= rep) {
+        const bf16* w = kind < rep ? qn : kn;
+        const float ss = warp_sum(x[0] * x[0] + x[1] * x[1] + x[2] * x[2] + x[3] * x[3]);
+        const float rstd = rsqrtf(ss / (float)kHD + p.eps);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] *= rstd * to_f(w[lane + 32 * e]);
+        const float* cs = p.rope + (size_t)(b * B + i) * (kHD / 2) * 2;
+        const float c0 = cs[2 * lane], s0 = cs[2 * lane + 1];
+        const float c1 = cs[2 * (lane + 32)], s1 = cs[2 * (lane + 32) + 1];
+        const float y0 = x[0] * c0 - x[2] * s0, y2 = x[2] * c0 + x[0] * s0;
+        const float y1 = x[1] * c1 - x[3] * s1, y3 = x[3] * c1 + x[1] * s1;
+        x[0] = y0; x[1] = y1; x[2] = y2; x[3] = y3;
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) dst[lane + 32 * e] = __float2bfloat16_rn(x[e]);
+    }
+  }
+  cp_async_wait_all();
+  __syncthreads();
+
+  // ---- online softmax over this warp's 16-key chunks
+  const int hh = warp / ksplit, ks = warp % ksplit;
+  const int nch_bw = nbw16 / 16;
+  const int nch = nch_bw + (p.R > 0 ? 1 : 0);
+  const float sl2 = 1.4426950408889634f * rsqrtf((float)kHD);
+  float rmax[2] = {-INFINITY, -INFINITY}, rsum[2] = {0.f, 0.f};
+  float o[16][4];
+#pragma unroll
+  for (int n = 0; n < 16; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  const bf16* qbase = sQ + (size_t)(hh * 16 + (lane & 15)) * row + (lane >> 4) * 8;
+
+  for (int c = ks; c < nch; c += ksplit) {
+    const bool summ = (c == nch_bw);
+    const bf16* Kc = summ ? sKs + (size_t)hh * 16 * row : sKbw + (size_t)c * 16 * row;
+    const bf16* Vc = summ ? sVs + (size_t)hh * 16 * row : sVbw + (size_t)c * 16 * row;
+    const int nvalid = summ ? p.R : min(16, nbw - c * 16);
+    float s[2][4];
+#pragma unroll
+    for (int n = 0; n < 2; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+    const bf16* kb = Kc + (size_t)((lane & 7) + (lane >> 4) * 8) * row + ((lane >> 3) & 1) * 8;
+#pragma unroll
+    for (int kk = 0; kk < kHD / 16; ++kk) {
+      uint32_t a[4], bk[4];
+      ldsm_x4(a, qbase + kk * 16);
+      ldsm_x4(bk, kb + kk * 16);
+      mma_bf16(s[0], a, bk[0], bk[1]);
+      mma_bf16(s[1], a, bk[2], bk[3]);
+    }
+#pragma unroll
+    for (int n = 0; n < 2; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (n * 8 + (lane & 3) * 2 + (e & 1) >= nvalid) s[n][e] = -INFINITY;
+    float mx0 = fmaxf(fmaxf(s[0][0], s[0][1]), fmaxf(s[1][0], s[1][1]));
+    float mx1 = fmaxf(fmaxf(s[0][2], s[0][3]), fmaxf(s[1][2], s[1][3]));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    const float n0 = fmaxf(rmax[0], mx0), n1 = fmaxf(rmax[1], mx1);
+    const float b0 = (n0 == -INFINITY) ? 0.f : n0, b1 = (n1 == -INFINITY) ? 0.f : n1;
+    const float sc0 = exp2f((rmax[0] - b0) * sl2), sc1 = exp2f((rmax[1] - b1) * sl2);
+    rmax[0] = n0;
+    rmax[1] = n1;
+    float pr[2][4];
+#pragma unroll
+    for (int n = 0; n < 2; ++n) {
+      pr[n][0] = exp2f((s[n][0] - b0) * sl2);
+      pr[n][1] = exp2f((s[n][1] - b0) * sl2);
+      pr[n][2] = exp2f((s[n][2] - b1) * sl2);
+      pr[n][3] = exp2f((s[n][3] - b1) * sl2);
+    }
+    rsum[0] = rsum[0] * sc0 + pr[0][0] + pr[0][1] + pr[1][0] + pr[1][1];
+    rsum[1] = rsum[1] * sc1 + pr[0][2] + pr[0][3] + pr[1][2] + pr[1][3];
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      o[n][0] *= sc0; o[n][1] *= sc0;
+      o[n][2] *= sc1; o[n][3] *= sc1;
+    }
+    uint32_t pa[4];
+    pa[0] = pack_bf16(pr[0][0], pr[0][1]);
+    pa[1] = pack_bf16(pr[0][2], pr[0][3]);
+    pa[2] = pack_bf16(pr[1][0], pr[1][1]);
+    pa[3] = pack_bf16(pr[1][2], pr[1][3]);
+    const bf16* vb = Vc + (size_t)((lane & 7) + ((lane >> 3) & 1) * 8) * row + (lane >> 4) * 8;
+#pragma unroll
+    for (int np = 0; np < kHD / 16; ++np) {
+      uint32_t bv[4];
+      ldsm_x4_t(bv, vb + np * 16);
+      mma_bf16(o[2 * np], pa, bv[0], bv[1]);
+      mma_bf16(o[2 * np + 1], pa, bv[2], bv[3]);
+    }
+  }
+  rsum[0] += __shfl_xor_sync(0xffffffffu, rsum[0], 1);
+  rsum[0] += __shfl_xor_sync(0xffffffffu, rsum[0], 2);
+  rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 1);
+  rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 2);
+
+  // ---- merge the key splits of each head (scratch reuses the K/V staging area)
+  __syncthreads();
+  float* scratch = reinterpret_cast<float*>(sKbw);
+  float* so = scratch + (size_t)warp * (16 * kHD + 32);
+  float* sml = so + 16 * kHD;
+  const int r0 = lane >> 2;
+#pragma unroll
+  for (int n = 0; n < 16; ++n) {
+    const int col = n * 8 + (lane & 3) * 2;
+    so[r0 * kHD + col] = o[n][0];
+    so[r0 * kHD + col + 1] = o[n][1];
+    so[(r0 + 8) * kHD + col] = o[n][2];
+    so[(r0 + 8) * kHD + col + 1] = o[n][3];
+  }
+  if ((lane & 3) == 0) {
+    sml[r0] = rmax[0];
+    sml[r0 + 8] = rmax[1];
+    sml[16 + r0] = rsum[0];
+    sml[16 + r0 + 8] = rsum[1];
+  }
+  __syncthreads();
+  bf16* out = static_cast<bf16*>(p.out);
+  const int ldo = p.nq * kHD;
+  for (int idx = tid; idx < rep * B * kHD; idx += nthr) {
+    const int e = idx % kHD, i = (idx / kHD) % B, h2 = idx / (kHD * B);
+    float M = -INFINITY;
+    for (int k = 0; k < ksplit; ++k) {
+      const float* ml = scratch + (size_t)(h2 * ksplit + k) * (16 * kHD + 32) + 16 * kHD;
+      M = fmaxf(M, ml[i]);
+    }
+    float num = 0.f, den = 0.f;
+    for (int k = 0; k < ksplit; ++k) {
+      const float* sw = scratch + (size_t)(h2 * ksplit + k) * (16 * kHD + 32);
+      const float f = exp2f((sw[16 * kHD + i] - M) * sl2);
+      den += f * sw[16 * kHD + 16 + i];
+      num += f * sw[i * kHD + e];
+    }
+    out[(size_t)(b * B + i) * ldo + (size_t)(g * rep + h2) * kHD + e] = __float2bfloat16_rn(num / den);
+  }
+}
+
+// ------------------------------------------------------------ fp32 reference shape
+template <typename T>
+__global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
+  extern __shared__ float ssm[];
+  const int d = p.d, B = p.B, half = d / 2;
+  const int rep = p.nq / p.nkv;
+  const int b = blockIdx.x / p.nq, h = blockIdx.x % p.nq, g = h / rep;
+  const long long t = p.t[b];
+  const int count = (int)(t < p.W ? t : p.W);
+  const int ctx = B + count + p.R;
+  float* sq = ssm;
+  float* sk = sq + B * d;
+  float* sv = sk + B * d;
+  float* ss = sv + B * d;                 // [B][ctx]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+  const T* qkv = static_cast<const T*>(p.qkv);
+  const int ldq = (p.nq + 2 * p.nkv) * d;
+  for (int item = warp; item < 3 * B; item += nw) {
+    const int i = item / 3, kind = item % 3;
+    const size_t mrow = (size_t)(b * B + i) * ldq;
+    const T* src = qkv + mrow + (kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
+                                                                      : (size_t)(p.nq + p.nkv + g) * d);
+    float* dst = (kind == 0 ? sq : kind == 1 ? sk : sv) + i * d;
+    if (kind == 2) {
+      for (int e = lane; e < d; e += 32) dst[e] = to_f(src[e]);
+      continue;
+    }
+    float part = 0.f;
+    for (int e = lane; e < d; e += 32) part += to_f(src[e]) * to_f(src[e]);
+    const float rstd = rsqrtf(warp_sum(part) / (float)d + p.eps);
+    const T* w = static_cast<const T*>(kind == 0 ? p.q_norm : p.k_norm);
+    const float* cs = p.rope + (size_t)(b * B + i) * half * 2;
+    for (int f = lane; f < half; f += 32) {
+      const float x1 = to_f(src[f]) * rstd * to_f(w[f]);
+      const float x2 = to_f(src[f + half]) * rstd * to_f(w[f + half]);
+      dst[f] = x1 * cs[2 * f] - x2 * cs[2 * f + 1];
+      dst[f + half] = x2 * cs[2 * f] + x1 * cs[2 * f + 1];
+    }
+  }
+  __syncthreads();
+  const size_t wbase = ((size_t)(b * p.L + p.layer) * p.nkv + g) * p.W * d;
+  const T* wk = static_cast<const T*>(p.win_k) + wbase;
+  const T* wv = static_cast<const T*>(p.win_v) + wbase;
+  const T* Gh = static_cast<const T*>(p.G) + ((size_t)p.layer * p.nq + h) * p.R * d;
+  const float* Mh = p.m + (((size_t)(b * p.L + p.layer) * p.nq + h) * p.R) * d;
+  const float scale = rsqrtf((float)d);
+  for (int idx = tid; idx < B * ctx; idx += blockDim.x) {
+    const int i = idx / ctx, j = idx % ctx;
+    float acc = 0.f;
+    if (j < B) {
+      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * sk[j * d + e];
+    } else if (j < B + count) {
+      const T* kr = wk + (size_t)(j - B) * d;
+      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * to_f(kr[e]);
+    } else {
+      const T* kr = Gh + (size_t)(j - B - count) * d;
+      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * to_f(kr[e]);
+    }
+    ss[idx] = acc * scale;
+  }
+  __syncthreads();
+  for (int i = warp; i < B; i += nw) {
+    float mx = -INFINITY;
+    for (int j = lane; j < ctx; j += 32) mx = fmaxf(mx, ss[i * ctx + j]);
+    mx = warp_max(mx);
+    float sum = 0.f;
+    for (int j = lane; j < ctx; j += 32) {
+      const float e = expf(ss[i * ctx + j] - mx);
+      ss[i * ctx + j] = e;
+      sum += e;
+    }
+    sum = warp_sum(sum);
+    for (int j = lane; j < ctx; j += 32) ss[i * ctx + j] /= sum;
+  }
+  __syncthreads();
+  T* out = static_cast<T*>(p.out);
+  for (int idx = tid; idx < B * d; idx += blockDim.x) {
+    const int i = idx / d, e = idx % d;
+    float acc = 0.f;
+    for (int j = 0; j < ctx; ++j) {
+      float v;
+      if (j < B) v = sv[j * d + e];
+      else if (j < B + count) v = to_f(wv[(size_t)(j - B) * d + e]);
+      else v = Mh[(size_t)(j - B - count) * d + e];
+      acc += ss[i * ctx + j] * v;
+    }
+    out[(size_t)(b * B + i) * p.nq * d + (size_t)h * d + e] = from_f<T>(acc);
+  }
+}
+
+int attn_ksplit(int B, int W, int nq, int nkv) {
+  const int rep = nq / nkv;
+  int ks = rep >= 16 ? 1 : 16 / rep;
+  while (ks > 1) {
+    AttnLayout a = attn_layout(B, W, nq, nkv, ks);
+    if (attn_merge_bytes(a.nwarps) <= a.bytes - a.off_kbw && a.nwarps <= 16) break;
+    --ks;
+  }
+  return ks;
+}
+
+size_t attn_smem_bytes(int B, int W, int nq, int nkv) {
+  AttnLayout a = attn_layout(B, W, nq, nkv, attn_ksplit(B, W, nq, nkv));
+  return a.bytes;
+}
+
+int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
+  if (dtype == LSP_DTYPE_BF16) {
+    if (p.d != kHD || p.B > 16 || p.R > 16) return LSP_ERR_SHAPE;
+    const int ks = attn_ksplit(p.B, p.W, p.nq, p.nkv);
+    AttnLayout a = attn_layout(p.B, p.W, p.nq, p.nkv, ks);
+    if (a.bytes > 227 * 1024 || attn_merge_bytes(a.nwarps) > a.bytes - a.off_kbw) return LSP_ERR_SHAPE;
+    static bool attr_set = false;
+    if (!attr_set) {
+      cudaFuncSetAttribute(attn_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      attr_set = true;
+    }
+    attn_mma_kernel<<<p.C * p.nkv, a.nwarps * 32, a.bytes, s>>>(p, a.rep, ks, a.rows_bw);
+  } else {
+    const int ctx = p.B + p.W + p.R;
+    const size_t smem = (size_t)(3 * p.B * p.d + p.B * ctx) * sizeof(float);
+    if (smem > 227 * 1024) return LSP_ERR_SHAPE;
+    static bool attr32 = false;
+    if (!attr32) {
+      cudaFuncSetAttribute(attn_simple_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           227 * 1024);
+      attr32 = true;
+    }
+    attn_simple_kernel<float><<<p.C * p.nq, 128, smem, s>>>(p);
+  }
+  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+}
+
+}  // namespace lsp

@@ -1,0 +1,139 @@
+// Internal host-side interfaces between the C-ABI layer and the kernel files.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/lsp.h"
+
+namespace lsp {
+
+// ------------------------------------------------------------------ GEMM
+enum EpiMode {
+  EPI_F32 = 0,     // Y (float) = acc
+  EPI_T = 1,       // Y (dtype) = acc
+  EPI_RESID = 2,   // Y (float) += acc
+  EPI_SWIGLU = 3,  // Y (dtype) = silu(acc_gate) * acc_up
+};
+
+constexpr int kGemmThreads = 192;   // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kTileRows = 128;      // weight rows per tile (UMMA M)
+
+struct GemmParams {
+  int M, N, K;          // token rows, output features, reduction length
+  int kblocks, splits, n_tiles;
+  int mode;
+  int seg_tile0[3];     // first tile index of each A segment
+  int nseg;
+  int bn, n_tok_tiles, m_pad, stages, tmem_cols;
+  void* Y;
+  int ldy;
+  float* ws;
+  int* counters;
+  unsigned* err;
+};
+
+struct GemmOp {
+  CUtensorMap a[3];
+  CUtensorMap b;
+  GemmParams p;
+  int dtype;
+  dim3 grid;
+  size_t smem;
+};
+
+// Plan Y = X W^T where W is the row-concatenation of `nseg` weight segments
+// (each [seg_rows[i]][K]); for EPI_SWIGLU, segment 0 = gate and 1 = up, both
+// [N][K].  splits <= 0 picks a split-K factor for `num_sms`.
+int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
+              const int* seg_rows, int nseg, int mode, void* Y, int ldy, float* ws,
+              size_t ws_bytes, int* counters, int n_counters, unsigned* err, int num_sms,
+              int splits);
+int gemm_launch(const GemmOp* op, cudaStream_t s);
+size_t gemm_ws_bytes(int M, int n_tiles, int splits);
+int gemm_tiles(int mode, const int* seg_rows, int nseg);
+int gemm_auto_splits(int n_tiles, int kblocks, int num_sms);
+
+// ------------------------------------------------------------------ view update
+struct ViewParams {
+  const void* k_new;
+  const void* v_new;
+  const void* h_new;
+  int rows;
+  const int32_t* acc;
+  const void* G;
+  void* win_k;
+  void* win_v;
+  float* m;
+  float* eta;
+  void* h;
+  int64_t* t;
+  int* done;
+  unsigned* err;
+  int C, L, nq, nkv, d, H, W, R;
+};
+int launch_view_update(const ViewParams& p, int dtype, cudaStream_t s);
+
+// ------------------------------------------------------------------ small ops
+struct CombineParams {
+  const int32_t* tokens;   // [C][B]
+  const void* embed;       // [V][H]
+  const void* pos;         // [B][H]
+  const void* mask_emb;    // [H]
+  const float* c;          // [C][H]
+  const void* norm_w;      // [H] first layer input norm
+  float* x;                // [M][H]
+  void* xn;                // [M][H]
+  float* rope;             // [C][B][d/2][2]
+  const int64_t* t;        // [C]
+  unsigned* err;
+  int C, B, H, V, d;
+  float eps;
+  double theta;
+};
+int launch_combine(const CombineParams& p, int dtype, cudaStream_t s);
+int launch_rmsnorm(const float* x, const void* w, void* out, int M, int H, float eps, int dtype,
+                   cudaStream_t s);
+
+// ------------------------------------------------------------------ attention
+struct AttnParams {
+  const void* qkv;        // [M][(nq+2nkv)d] projections (pre-norm, pre-rotary)
+  const void* q_norm;     // [d]
+  const void* k_norm;     // [d]
+  const float* rope;      // [C][B][d/2][2]
+  const void* win_k;      // state window of the tapped layer's base: [C][L][nkv][W][d]
+  const void* win_v;
+  const void* G;          // [L][nq][R][d]
+  const float* m;         // [C][L][nq][R][d]
+  const int64_t* t;       // [C]
+  void* out;              // [M][nq d]
+  int C, B, L, nq, nkv, d, W, R, layer;
+  float eps;
+};
+int launch_attention(const AttnParams& p, int dtype, cudaStream_t s);
+
+// ------------------------------------------------------------------ sampler
+struct SampleParams {
+  const float* src;       // [C][B][V] base logits
+  float* dst;             // [C][B][V] corrected logits or nullptr
+  const int32_t* prev;    // y_0 source: element b * prev_stride
+  int prev_stride;
+  const void* Ec;
+  const void* Wc;
+  int32_t* out_tokens;    // [C][B]
+  float* part_val;        // [2][nblk][C]
+  int* part_idx;          // [2][nblk][C]
+  unsigned* err;
+  int C, B, V, rc, nblk;
+  float temperature;
+  uint32_t round;
+  uint64_t seed;
+};
+int sample_blocks(int num_sms);
+int launch_sample(const SampleParams& p, int dtype, cudaStream_t s);
+int launch_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint32_t* out,
+                        int count, cudaStream_t s);
+
+}  // namespace lsp

@@ -1,0 +1,137 @@
+"""Full drafting round on the GPU (lsp_view_update + lsp_draft) vs the fp64 oracle.
+
+Tolerances (bf16 path): row-wise max |z_gpu - z_oracle| / max |z_oracle| <= 2e-2;
+the fp32-storage shape (tf32 tensor cores) <= 5e-3.  Tokens must be bit-exact at
+every position whose oracle top-1/top-2 margin of the decision score exceeds
+1e-2, with the oracle teacher-forced on the GPU's previous token.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_37029_gb300 import synth
+from tests.gpu_common import cuda_weights, f64, fold_chunk, lsp_lib, np_weights
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"bf16": 2e-2, "f32": 5e-3}
+
+
+@pytest.fixture(scope="module")
+def lsp():
+    return lsp_lib()
+
+
+def _compare(s, z_gpu, toks_gpu, z0_orc, ow, bt, temperature, seed, rnd, reqs):
+    checked = total = 0
+    worst = 0.0
+    for r, b in enumerate(reqs):
+        t_o, z_o, marg = oracle.sample_block(z0_orc[r], int(bt[b, 0]), ow.Ec, ow.Wc, temperature,
+                                             seed, rnd, b, forced_prev=toks_gpu[b])
+        for i in range(s.B):
+            rel = np.abs(z_gpu[b, i] - z_o[i]).max() / np.abs(z_o[i]).max()
+            worst = max(worst, rel)
+        sel = marg > 1e-2
+        assert np.array_equal(toks_gpu[b][sel], t_o[sel]), (b, toks_gpu[b], t_o, marg)
+        checked += int(sel.sum())
+        total += s.B
+    assert worst <= TOL[s.dtype], worst
+    assert checked >= 0.5 * total, (checked, total)      # guard against a vacuous comparison
+    return worst
+
+
+def _run_round(lsp, s, prefix, reqs=None, chunk=1024, device_gen=False):
+    """Fold a synthetic prefix and one round into both sides, draft, compare."""
+    reqs = list(range(s.C)) if reqs is None else reqs
+    so = s.with_(C=len(reqs))                 # oracle shape: the sampled requests only
+    gdev = "cuda" if device_gen else "cpu"
+    w = synth.make_weights(s, device=gdev)
+    wc = cuda_weights(w) if not device_gen else w
+    ow = oracle.OracleWeights(np_weights(w))
+    st = lsp.lsp_state_create(lsp.make_config(s))
+    try:
+        lsp.lsp_state_init(st, wc["G"])
+        ost = oracle.state_init(so)
+        base = synth.input_seed(s) * 1000
+        for c0 in range(0, prefix, chunk):
+            n = min(chunk, prefix - c0)
+            k, v, h = synth.make_features(s, n, seed=base + c0 // chunk, device=gdev)
+            acc = torch.full((s.C,), n, dtype=torch.int32)
+            lsp.lsp_view_update(st, k.cuda(), v.cuda(), h.cuda(), acc.cuda())
+            oracle.view_update(so, ost, ow.G, f64(k[reqs]), f64(v[reqs]), f64(h[reqs]), acc[reqs].numpy())
+        k, v, h = synth.make_features(s, s.B + 1, seed=base + 999, device=gdev)
+        acc = synth.make_accepted(s, seed=base + 998, hi=min(s.delta_max, s.B + 1))
+        acc[0] = s.B + 1                                   # one request accepts the whole block
+        if s.C > 2:
+            acc[1] = 0                                     # and one accepts nothing new
+        lsp.lsp_view_update(st, k.cuda(), v.cuda(), h.cuda(), acc.cuda())
+        oracle.view_update(so, ost, ow.G, f64(k[reqs]), f64(v[reqs]), f64(h[reqs]), acc[reqs].numpy())
+        bt = synth.make_block_tokens(s, seed=base + 997)
+        toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
+        z = torch.zeros(s.C, s.B, s.V, device="cuda")
+        sp = lsp.make_sample_params(s.temperature, seed=synth.RNG_SEED, rnd=3)
+        lsp.lsp_draft(st, bt.cuda(), lsp.make_weights(wc), sp, toks, z)
+        torch.cuda.synchronize()
+        assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+        toks_g = toks.cpu().numpy()
+        z_g = z.cpu().double().numpy()
+        z0 = oracle.draft_base_logits(so, ost, ow, bt[reqs].numpy())
+        bt_np = bt.numpy()
+        z0_full = {b: z0[r] for r, b in enumerate(reqs)}
+        return _compare(s, z_g, toks_g, [z0_full[b] for b in reqs], ow, bt_np, s.temperature,
+                        synth.RNG_SEED, 3, reqs)
+    finally:
+        lsp.lsp_state_destroy(st)
+
+
+@pytest.mark.parametrize("name", ["tiny", "small"])
+def test_round_matches_oracle(lsp, name):
+    s = synth.SHAPES[name]
+    _run_round(lsp, s, s.prefix)
+
+
+def test_round_sampled_and_short_prefix(lsp):
+    """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
+    s = synth.SMALL.with_(temperature=1.0)
+    _run_round(lsp, s, 100)
+
+
+def test_round_is_deterministic_and_reports_bad_tokens(lsp):
+    s = synth.SMALL
+    w = cuda_weights(synth.make_weights(s))
+    st = lsp.lsp_state_create(lsp.make_config(s))
+    try:
+        lsp.lsp_state_init(st, w["G"])
+        k, v, h = synth.make_features(s, 600, seed=1, device="cuda")
+        lsp.lsp_view_update(st, k, v, h, torch.full((s.C,), 600, dtype=torch.int32, device="cuda"))
+        bt = synth.make_block_tokens(s, seed=2).cuda()
+        ws = lsp.make_weights(w)
+        sp = lsp.make_sample_params(1.0, seed=5, rnd=1)
+        outs = []
+        for _ in range(2):
+            toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
+            z = torch.zeros(s.C, s.B, s.V, device="cuda")
+            lsp.lsp_draft(st, bt, ws, sp, toks, z)
+            outs.append((toks.clone(), z.clone()))
+        assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+        # without out_logits the tokens are the same
+        toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
+        lsp.lsp_draft(st, bt, ws, sp, toks, None)
+        assert torch.equal(toks, outs[0][0])
+        assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+        bad = bt.clone()
+        bad[1, 3] = s.V
+        lsp.lsp_draft(st, bad, ws, sp, toks, None)
+        rc, bits = lsp.lsp_get_error(st)
+        assert bits == lsp.LSP_DEV_BAD_TOKEN
+    finally:
+        lsp.lsp_state_destroy(st)
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["qwen3-8b", "large"])
+def test_full_size_round_on_sampled_requests(lsp, name):
+    """Full shapes (C=16 / C=32, V=151936) at a 4K prefix, oracle on two requests."""
+    s = synth.SHAPES[name]
+    _run_round(lsp, s, 4096, reqs=[0, s.C - 1], chunk=2048, device_gen=True)
