@@ -1,0 +1,572 @@
+#!/usr/bin/env python
+"""Benchmark of the fixed-cost drafting round on one GB300 (or N replicas).
+
+One step = one drafting round over all C requests: lsp_view_update (fold the
+new target rows into the fixed-size interface) + lsp_draft (boundary fusion,
+D draft layers, LM head, Markov correction + sampling of B proposals).
+
+Default workload: Qwen3-8B-shaped drafter at concurrency 16, 32K-token prefix,
+temperature-1 sampling (C=16, B=16, L=5 tapped layers, D=5, H=4096, 32 q / 8 kv
+heads x 128, MLP 12288, V=151936, W=256, R=16).  All inputs are seeded
+synthetic tensors (see paper_2609_37029_gb300/synth.py); weights are random
+init.  The 3.3 GB of projection weights streamed every round exceed the
+129 MB L2, so no explicit flush is needed between timed rounds.
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 oracle on
+the host cores instead (the baseline of this tier).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np
+import torch
+
+from paper_2609_37029_gb300 import synth
+
+METRIC = "drafting µs/round and drafted tokens/s vs prefix length at concurrency 16; % roofline"
+UNIT = "drafted tokens/s"
+FOLD_CHUNK = 2048
+GEMM_STAGES = ("fuse", "qkv", "o_proj", "gate_up", "down", "lm_head")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="qwen3-8b", choices=sorted(synth.SHAPES))
+    ap.add_argument("--prefix", type=int, default=None)
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=150.0, help="seconds for the oracle legs")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ distributed plumbing
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            torch.cuda.set_device(self.local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", self.local))
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        t = torch.tensor([x], device="cuda", dtype=torch.float64)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ------------------------------------------------------------------ clocks during the timed region
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self):
+        self.proc = None
+        self.target = self._gpu_id()
+
+    @staticmethod
+    def _gpu_id():
+        try:
+            p = torch.cuda.get_device_properties(torch.cuda.current_device())
+            return f"{p.pci_domain_id:08X}:{p.pci_bus_id:02X}:{p.pci_device_id:02X}.0"
+        except Exception:
+            vis = os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0]
+            return vis or "0"
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.target}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        self.proc.terminate()
+        try:
+            out = self.proc.communicate(timeout=10)[0]
+        except Exception:
+            self.proc.kill()
+            out = ""
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------ algorithmic work
+def gemm_work(s, name):
+    """(bytes, flops) of one projection launch: weights + activations in + outputs out."""
+    es = 2 if s.dtype == "bf16" else 4
+    M = s.C * s.B
+    if name == "fuse":
+        Mx, N, K, out = s.C, s.H, s.L * s.H, s.C * s.H * 4
+    elif name == "qkv":
+        Mx, N, K = M, (s.nq + 2 * s.nkv) * s.d, s.H
+        out = M * N * es
+    elif name == "o_proj":
+        Mx, N, K = M, s.H, s.nq * s.d
+        out = 2 * M * N * 4                      # residual read + write
+    elif name == "gate_up":
+        Mx, N, K = M, 2 * s.F, s.H
+        out = M * s.F * es
+    elif name == "down":
+        Mx, N, K = M, s.H, s.F
+        out = 2 * M * N * 4
+    else:                                        # lm_head
+        Mx, N, K = M, s.V, s.H
+        out = M * N * 4
+    return N * K * es + Mx * K * es + out, 2.0 * Mx * N * K
+
+
+def round_work(s, mean_delta):
+    """Algorithmic bytes / flops of one round: weights once, interface state touched, one logits write."""
+    es = 2 if s.dtype == "bf16" else 4
+    nb = 0
+    fl = 0.0
+    names = ["fuse"] + ["qkv", "o_proj", "gate_up", "down"] * s.D + ["lm_head"]
+    for n in names:
+        b, f = gemm_work(s, n)
+        nb += b
+        fl += f
+    kv = s.nkv * s.d
+    # view update: new K/V rows read + window write, summary (m, eta) read+write, G, boundary
+    nb += s.C * mean_delta * s.L * 2 * kv * es * 2
+    nb += 2 * s.C * s.L * s.nq * s.R * (s.d + 1) * 4 + s.L * s.nq * s.R * s.d * es + s.C * s.L * s.H * es
+    fl += 4.0 * s.C * s.L * s.nq * s.R * mean_delta * s.d
+    # attention: window K/V + summary values per draft layer
+    ctx = s.B + s.W + s.R
+    nb += s.C * s.D * (s.W * 2 * kv * es + s.nq * s.R * s.d * 4)
+    fl += 4.0 * s.C * s.D * s.nq * s.B * ctx * s.d
+    # correction factors and the sampler's corrected-logit pass
+    nb += 2 * s.V * s.rc * es
+    fl += 2.0 * s.C * s.B * s.V * s.rc
+    return nb, fl
+
+
+def launches_per_round(s):
+    return 1 + 1 + 1 + 7 * s.D + 1 + (s.B + 1)
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), float(j["bf16_tflops"]), float(j["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def profiled_traffic(kernel_file, workload):
+    """DRAM bytes per launch from a committed ncu summary, if taken on the current source."""
+    path = os.path.join(ROOT, "profiles", f"{kernel_file}_{workload}.md")
+    src = os.path.join(ROOT, "paper_2609_37029_gb300", "csrc", kernel_file.split("__")[0] + ".cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        txt = open(path).read()
+    except OSError:
+        return None
+    vals = {}
+    for line in txt.splitlines():
+        if line.startswith("traffic_key:"):
+            k, v = line.split(":", 1)[1].split("=")
+            vals[k.strip()] = v.strip()
+    if vals.get("source_sha256_16") != sha:
+        return None
+    try:
+        return float(vals["dram_bytes_per_round"])
+    except (KeyError, ValueError):
+        return None
+
+
+# ------------------------------------------------------------------ workload
+class Workload:
+    def __init__(self, s, lsp, seed_base):
+        self.s, self.lsp = s, lsp
+        self.seed_base = seed_base
+        self.w = synth.make_weights(s, seed=synth.WEIGHT_SEED, device="cuda")
+        self.ws = lsp.make_weights(self.w)
+        self.cfg = lsp.make_config(s)
+        rows = s.B + 1
+        self.k, self.v, self.h = synth.make_features(s, rows, seed=seed_base + 5000, device="cuda")
+        self.acc = synth.make_accepted(s, seed=seed_base + 5001, device="cuda")
+        self.bt = synth.make_block_tokens(s, seed=seed_base + 5002, device="cuda")
+        self.toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
+        self.logits = torch.empty(s.C, s.B, s.V, device="cuda")
+        self.sp = lsp.make_sample_params(s.temperature, seed=synth.RNG_SEED, rnd=0)
+        self._hfold = None
+
+    def new_state(self):
+        st = self.lsp.lsp_state_create(self.cfg)
+        self.lsp.lsp_state_init(st, self.w["G"])
+        return st
+
+    def fold(self, st, start, end, keep=None):
+        """Fold prefix rows [start, end) in FOLD_CHUNK-row chunks (GPU-generated, seeded)."""
+        s = self.s
+        if self._hfold is None:
+            _, _, self._hfold = synth.make_features(s, FOLD_CHUNK, seed=self.seed_base + 7000, device="cuda")
+        for c0 in range(start, end, FOLD_CHUNK):
+            n = min(FOLD_CHUNK, end - c0)
+            k, v, _ = synth.make_features(s, FOLD_CHUNK, seed=self.seed_base + c0 // FOLD_CHUNK,
+                                          device="cuda", with_h=False)
+            acc = torch.full((s.C,), n, dtype=torch.int32, device="cuda")
+            self.lsp.lsp_view_update(st, k, v, self._hfold, acc, rows=FOLD_CHUNK)
+            if keep is not None:
+                keep.append((k[0:1, :, :n].cpu(), v[0:1, :, :n].cpu(),
+                             self._hfold[0:1, :, n - 1:n].cpu()))
+
+    def round(self, st):
+        self.lsp.lsp_view_update(st, self.k, self.v, self.h, self.acc)
+        self.lsp.lsp_draft(st, self.bt, self.ws, self.sp, self.toks, self.logits)
+
+    def capture(self, st):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.round(st)
+        return g
+
+
+def time_graph(g, steps, warmup, dist, clocks=None):
+    if clocks:
+        clocks.start()                  # samples span the warm-up and the timed replays
+    for _ in range(warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    dist.barrier()
+    ck = clocks.stop() if clocks else None
+    return e0.elapsed_time(e1) / steps, ck
+
+
+def stage_times(wl, st, reps):
+    """Per-stage device time of a captured round via the library's stage-event hook."""
+    lsp = wl.lsp
+    n = lsp.lsp_stage_count(st)
+    names = [lsp.lsp_stage_name(st, k) for k in range(n)]
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    for e in evs:
+        e.record()
+    torch.cuda.synchronize()
+    lsp.lsp_set_stage_events(st, evs)
+    try:
+        g = wl.capture(st)
+        run = g.replay
+    except Exception:                    # event nodes not capturable here: time eager rounds
+        g = None
+        run = lambda: wl.round(st)
+    acc = np.zeros(n)
+    try:
+        for _ in range(3):
+            run()
+        torch.cuda.synchronize()
+        for _ in range(reps):
+            run()
+            torch.cuda.synchronize()
+            acc += [evs[k].elapsed_time(evs[k + 1]) for k in range(n)]
+    finally:
+        lsp.lsp_set_stage_events(st, [])
+    return names, acc / reps
+
+
+# ------------------------------------------------------------------ oracle (CPU) legs
+def oracle_weights(w):
+    import oracle
+
+    def host64(t):
+        return t.detach().to(torch.float64).cpu().numpy()
+
+    wn = {k: host64(v) for k, v in w.items() if k not in ("layers", "embed")}
+    wn["embed"] = w["embed"].detach().float().cpu().numpy()       # rows gathered on use
+    wn["layers"] = [{k: host64(v) for k, v in lw.items()} for lw in w["layers"]]
+    return oracle.OracleWeights(wn)
+
+
+def oracle_prefix_state(s1, ow, kept):
+    """Oracle interface of request 0 after the same prefix the GPU folded."""
+    import oracle
+    ost = oracle.state_init(s1)
+    for k, v, hlast in kept:
+        n = k.shape[2]
+        h = np.zeros((1, s1.L, n, s1.H))
+        h[:, :, n - 1] = hlast[:, :, 0].double().numpy()
+        oracle.view_update(s1, ost, ow.G, k.double().numpy(), v.double().numpy(), h, np.array([n]))
+    return ost
+
+
+def oracle_round(s1, ow, ost, wl):
+    """Request 0's share of one round, as the oracle computes it; returns seconds."""
+    import oracle
+    t0 = time.perf_counter()
+    oracle.view_update(s1, ost, ow.G, wl.k[0:1].double().cpu().numpy(), wl.v[0:1].double().cpu().numpy(),
+                       wl.h[0:1].double().cpu().numpy(), wl.acc[0:1].cpu().numpy())
+    bt = wl.bt[0:1].cpu().numpy()
+    z0 = oracle.draft_base_logits(s1, ost, ow, bt)
+    oracle.sample_block(z0[0], int(bt[0, 0]), ow.Ec, ow.Wc, s1.temperature, synth.RNG_SEED, 0, 0)
+    return time.perf_counter() - t0
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_leg(wl, kept, budget, max_steps=None, warmup=1):
+    s = wl.s
+    s1 = s.with_(C=1)
+    ow = oracle_weights(wl.w)
+    ost = oracle_prefix_state(s1, ow, kept)
+    for _ in range(warmup):
+        oracle_round(s1, ow, ost, wl)
+    times = []
+    t_start = time.perf_counter()
+    while True:
+        times.append(oracle_round(s1, ow, ost, wl))
+        if max_steps is not None and len(times) >= max_steps:
+            break
+        if time.perf_counter() - t_start > budget or (max_steps is None and sum(times) > 10.0):
+            break
+    t_req = statistics.mean(times)
+    return {"value": s.B / t_req, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+            "sample": (f"request 0 of {s.C}: its view update (accepted_len new rows), drafter forward "
+                       f"and {s.B}-step correction+sampling in numpy fp64, repeated {len(times)}x "
+                       f"after {warmup} warm-up; round time = {s.C} x sample ({t_req:.2f} s)"),
+            "_t_req": t_req, "_steps": len(times)}
+
+
+# ------------------------------------------------------------------ main
+def workload_config(s, prefix):
+    return {"workload": (f"{s.name} drafting round: C={s.C}, B={s.B}, {s.L} tapped layers, D={s.D}, "
+                         f"H={s.H}, {s.nq}q/{s.nkv}kv x {s.d}, F={s.F}, V={s.V}, W={s.W}, R={s.R}, "
+                         f"r_c={s.rc}, prefix {prefix}, "
+                         + ("greedy" if s.temperature == 0 else f"T={s.temperature:g} sampling")),
+            "C": s.C, "B": s.B, "prefix": prefix, "global_batch": s.C, "seq_len": prefix,
+            "parallelism": "replicas", "accepted_len": f"U[1,{s.delta_max}] seeded",
+            "l2": "no flush: >3 GB of weights streamed per round exceed the 129 MB L2"}
+
+
+def run_reference(args, dist):
+    if dist.rank != 0:
+        return
+    from paper_2609_37029_gb300 import build as _b
+    _b.build()
+    from paper_2609_37029_gb300 import lsp
+    s = synth.SHAPES[args.config]
+    prefix = args.prefix or s.prefix
+    wl = Workload(s, lsp, synth.input_seed(s) * 1000)
+    st = wl.new_state()
+    kept = []
+    wl.fold(st, 0, prefix, keep=kept)
+    torch.cuda.synchronize()
+    lsp.lsp_state_destroy(st)
+    leg = oracle_leg(wl, kept, args.cpu_budget, max_steps=max(1, args.steps),
+                     warmup=min(args.warmup, 1))
+    ms = leg["_t_req"] * s.C * 1e3
+    out = {"impl": "reference", "metric": METRIC, "value": leg["value"], "unit": UNIT,
+           "n_gpus": args.gpus, "steps": leg["_steps"], "warmup": min(args.warmup, 1),
+           "ms_per_step": ms, "us_per_round": ms * 1e3, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": workload_config(s, prefix),
+           "cpu_baseline": {k: v for k, v in leg.items() if not k.startswith("_")},
+           "e2e": {"value": leg["value"], "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0},
+           "note": "steps capped by the time budget; each step is one request's share of a round"}
+    print(json.dumps(out), flush=True)
+
+
+def run_ours(args, dist):
+    from paper_2609_37029_gb300 import build as _b
+    if dist.local == 0:
+        _b.build()
+    dist.barrier()
+    from paper_2609_37029_gb300 import lsp
+    torch.cuda.set_device(dist.local)
+    s = synth.SHAPES[args.config]
+    prefix = args.prefix or s.prefix
+    hbm, tf_burst, tf_sust, peak_src = peaks()
+    wl = Workload(s, lsp, synth.input_seed(s) * 1000)
+    st = wl.new_state()
+    want_cpu = dist.rank == 0 and dist.world == 1 and not args.no_cpu
+    kept = [] if want_cpu else None
+    wl.fold(st, 0, prefix, keep=kept)
+    for _ in range(2):
+        wl.round(st)
+    torch.cuda.synchronize()
+    rc, bits = lsp.lsp_get_error(st)
+    if rc != lsp.LSP_OK:
+        raise RuntimeError(f"device error after warm-up: {rc} bits={bits}")
+    g = wl.capture(st)
+    ms, clocks = time_graph(g, args.steps, args.warmup, dist, Clocks())
+    ms = dist.max(ms)
+    rc, bits = lsp.lsp_get_error(st)
+    if rc != lsp.LSP_OK:
+        raise RuntimeError(f"device error in the timed region: {rc} bits={bits}")
+
+    # per-stage device times (dominant kernel = the projection GEMM)
+    names, st_ms = stage_times(wl, st, reps=min(200, max(20, args.steps // 5)))
+    gemm_bytes = gemm_flops = gemm_ms = 0.0
+    stages = {}
+    for n, t in zip(names, st_ms):
+        stages[n] = stages.get(n, 0.0) + float(t) * 1e3
+        if n in GEMM_STAGES:
+            b, f = gemm_work(s, n)
+            gemm_bytes += b
+            gemm_flops += f
+            gemm_ms += float(t)
+    n_gemm = sum(1 for n in names if n in GEMM_STAGES)
+    ach = gemm_bytes / (gemm_ms * 1e-3) / 1e9
+    intensity = gemm_flops / gemm_bytes
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    traffic_round = profiled_traffic("k_gemm", s.name)
+    roofline = {"bound": "hbm" if intensity < ridge else "tensor",
+                "kernel": f"gemm_kernel (tcgen05 projection GEMM, {n_gemm} launches per round)",
+                "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+                "peak_source": f"{peak_src} HBM copy bandwidth",
+                "traffic": (traffic_round / n_gemm) if traffic_round else None,
+                "algorithmic_bytes_per_launch": gemm_bytes / n_gemm,
+                "avg_launch_us": gemm_ms * 1e3 / n_gemm,
+                "tensor_tflops": gemm_flops / (gemm_ms * 1e-3) / 1e12,
+                "tensor_frac_of_sustained": gemm_flops / (gemm_ms * 1e-3) / 1e12 / tf_sust,
+                "intensity_flop_per_byte": intensity}
+    mean_delta = float(wl.acc.float().mean())
+    rb, rf = round_work(s, mean_delta)
+    t_roof = max(rb / (hbm * 1e9), rf / (tf_burst * 1e12))
+    round_roof = {"bytes": rb, "flops": rf, "roofline_us": t_roof * 1e6,
+                  "frac": t_roof * 1e3 / ms}
+
+    # end to end through the C ABI with host buffers (pinned), copies inside the timed region
+    hk, hv, hh = wl.k.cpu().pin_memory(), wl.v.cpu().pin_memory(), wl.h.cpu().pin_memory()
+    hacc, hbt = wl.acc.cpu().pin_memory(), wl.bt.cpu().pin_memory()
+    htoks = torch.empty(s.C, s.B, dtype=torch.int32).pin_memory()
+
+    def e2e_step():
+        wl.k.copy_(hk, non_blocking=True)
+        wl.v.copy_(hv, non_blocking=True)
+        wl.h.copy_(hh, non_blocking=True)
+        wl.acc.copy_(hacc, non_blocking=True)
+        wl.bt.copy_(hbt, non_blocking=True)
+        wl.round(st)
+        htoks.copy_(wl.toks, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    k_e = min(args.steps, 300)
+    for _ in range(min(args.warmup, 10)):
+        e2e_step()
+    dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(k_e):
+        e2e_step()
+    e2e_ms = dist.max((time.perf_counter() - t0) * 1e3 / k_e)
+    h2d = sum(t.numel() * t.element_size() for t in (hk, hv, hh, hacc, hbt))
+    d2h = htoks.numel() * htoks.element_size()
+
+    # prefix sweep: drafting time and state bytes vs prefix length
+    sweep = None
+    prefixes = synth.SWEEP.prefixes if s.name in ("qwen3-8b", "qwen3-8b-sweep") else ()
+    if prefixes and not args.no_sweep:
+        st2 = wl.new_state()
+        done = 0
+        pts = {}
+        for p in prefixes:
+            wl.fold(st2, done, p)
+            done = p
+            g2 = wl.capture(st2)
+            m2, _ = time_graph(g2, max(100, args.steps // 4), 10, dist)
+            pts[str(p)] = dist.max(m2) * 1e3
+            del g2
+        vals = list(pts.values())
+        sweep = {"us_per_round": pts, "max_over_min": max(vals) / min(vals),
+                 "state_bytes": lsp.lsp_state_bytes(wl.cfg), "state_bytes_constant": True}
+        lsp.lsp_state_destroy(st2)
+
+    cpu = None
+    if want_cpu:
+        leg = oracle_leg(wl, kept, args.cpu_budget)
+        cpu = {k: v for k, v in leg.items() if not k.startswith("_")}
+
+    value = dist.world * s.C * s.B / (ms * 1e-3)
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "us_per_round": ms * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
+           "data": "synthetic (seeded random features and random-init weights)",
+           "config": workload_config(s, prefix),
+           "roofline": roofline, "round_roofline": round_roof,
+           "stages_us": {k: round(v, 2) for k, v in stages.items()},
+           "e2e": {"value": dist.world * s.C * s.B / (e2e_ms * 1e-3), "unit": UNIT,
+                   "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+           "gpu_launches": launches_per_round(s) * args.steps,
+           "clocks": clocks, "sweep": sweep, "cpu_baseline": cpu}
+    if dist.rank == 0:
+        print(json.dumps(out), flush=True)
+    lsp.lsp_state_destroy(st)
+
+
+def main():
+    args = parse_args()
+    dist = Dist()
+    try:
+        if args.impl == "reference":
+            run_reference(args, dist)
+        else:
+            run_ours(args, dist)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -87,8 +87,9 @@ struct lsp_state {
 namespace {
 const char* kLayerStages[7] = {"qkv", "attention", "o_proj", "post_norm", "gate_up", "down", "next_norm"};
 inline int stage_total(const lsp_config& c) { return 5 + 7 * c.D; }
+// External records so that a captured round carries them as event-record nodes.
 inline void mark(lsp_state* st, int k, cudaStream_t s) {
-  if (k < st->n_stage_ev) cudaEventRecord(st->stage_ev[k], s);
+  if (k < st->n_stage_ev) cudaEventRecordWithFlags(st->stage_ev[k], s, cudaEventRecordExternal);
 }
 }  // namespace
 
