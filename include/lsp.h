@@ -217,6 +217,29 @@ int lsp_sample(lsp_state* st, const float* base_logits, const int32_t* prev_toke
                const void* Ec, const void* Wc, const lsp_sample_params* sp,
                int32_t* out_tokens, float* out_logits, lsp_stream_t stream);
 
+/* Correction + sampling without a state and without any device allocation,
+ * for callers that cannot allocate device memory where they sample (a loop
+ * running under another framework's caching allocator that already reserved
+ * the device, or code that must not create an lsp_state).  The paper has no
+ * counterpart: this is a deployment variant of lsp_sample.
+ *   Same computation and tensor arguments as lsp_sample; the shapes are passed
+ *   explicitly (1 <= C <= 64, B >= 1, V and rc multiples of 16, rc <= 256) and
+ *   dtype is LSP_DTYPE_BF16 or LSP_DTYPE_F32 for Ec / Wc.
+ *   dev_error: optional device uint32 that receives LSP_DEV_* bits (OR-ed in;
+ *   NULL skips error reporting).
+ * Scratch: a fixed 512 KiB __device__ array inside the library, held by every
+ * GPU that loads it until the process exits; a call needs 16 * (2 * SMs) * C
+ * bytes of it and returns LSP_ERR_SHAPE beyond that.  The first call on a
+ * device looks up the array's device address and the SM count; make that
+ * first call before any stream capture on the device.  Every call shares the
+ * array: calls that overlap on the GPU (other streams or threads) race, so
+ * the caller must serialise them.  Allocates nothing and calls no allocating
+ * CUDA or library routine. */
+int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, const void* Ec,
+                       const void* Wc, int dtype, int C, int B, int V, int rc,
+                       const lsp_sample_params* sp, int32_t* out_tokens, float* out_logits,
+                       uint32_t* dev_error, lsp_stream_t stream);
+
 /* Dense projection Y = X W^T with the drafter's tensor-core GEMM (the kernel
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].

@@ -1,0 +1,95 @@
+// lsp_sample_noalloc: the correction + sampling step for callers that cannot
+// allocate device memory.
+//
+// Some callers of this library cannot call cudaMalloc at the point where they
+// sample: a serving loop that runs inside a custom allocator's critical
+// section, a process whose device memory is fully reserved by another
+// framework's caching allocator, or code that must not create a state object
+// (lsp_state_create allocates the interface and a workspace).  The sampler's
+// only scratch is the per-CTA argmax partials of two consecutive steps, so this
+// variant keeps them in a fixed file-scope __device__ array instead.  Every GPU
+// that loads the library holds that array until the process exits.
+#include <cmath>
+#include <mutex>
+
+#include "lsp_internal.h"
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = 512 * 1024;     // the documented maximum (512 KiB)
+constexpr int kMaxDevices = 64;
+
+__device__ __align__(256) unsigned char g_sample_scratch[kStaticScratchBytes];
+
+struct DeviceScratch {
+  std::once_flag once;
+  int status = LSP_ERR_CUDA;
+  unsigned char* ptr = nullptr;     // device address of g_sample_scratch on this device
+  int num_sms = 0;
+};
+DeviceScratch g_dev[kMaxDevices];
+
+// Once per device, with that device current: the device address of the array
+// (the host-side symbol is only a stand-in) and the SM count.
+int scratch_for_current_device(DeviceScratch** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return LSP_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return LSP_ERR_UNSUPPORTED;
+  DeviceScratch& ds = g_dev[dev];
+  std::call_once(ds.once, [&ds, dev] {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_sample_scratch) != cudaSuccess) {
+      ds.status = LSP_ERR_CUDA;
+      return;
+    }
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) {
+      ds.status = LSP_ERR_CUDA;
+      return;
+    }
+    ds.ptr = static_cast<unsigned char*>(p);
+    ds.num_sms = sms;
+    ds.status = LSP_OK;
+  });
+  *out = &ds;
+  return ds.status;
+}
+
+}  // namespace
+
+extern "C" int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token,
+                                  const void* Ec, const void* Wc, int dtype, int C, int B, int V,
+                                  int rc, const lsp_sample_params* sp, int32_t* out_tokens,
+                                  float* out_logits, uint32_t* dev_error, lsp_stream_t stream) {
+  if (!base_logits || !prev_token || !Ec || !Wc || !sp || !out_tokens) return LSP_ERR_ARG;
+  if (dtype != LSP_DTYPE_BF16 && dtype != LSP_DTYPE_F32) return LSP_ERR_ARG;
+  if (!(sp->temperature >= 0.f) || !std::isfinite(sp->temperature)) return LSP_ERR_ARG;
+  if (C < 1 || C > 64 || B < 1 || V < 16 || V % 16 || rc < 16 || rc % 16 || rc > 256)
+    return LSP_ERR_SHAPE;
+  DeviceScratch* ds = nullptr;
+  int rc_setup = scratch_for_current_device(&ds);
+  if (rc_setup != LSP_OK) return rc_setup;
+  const int nblk = lsp::sample_blocks(ds->num_sms);
+  const size_t part = (size_t)2 * nblk * C;                  // values, then indices
+  if (part * (sizeof(float) + sizeof(int)) > kStaticScratchBytes) return LSP_ERR_SHAPE;
+  lsp::SampleParams p;
+  p.src = base_logits;
+  p.dst = out_logits;
+  p.prev = prev_token;
+  p.prev_stride = 1;
+  p.Ec = Ec;
+  p.Wc = Wc;
+  p.out_tokens = out_tokens;
+  p.part_val = reinterpret_cast<float*>(ds->ptr);
+  p.part_idx = reinterpret_cast<int*>(ds->ptr + part * sizeof(float));
+  p.err = reinterpret_cast<unsigned*>(dev_error);
+  p.C = C;
+  p.B = B;
+  p.V = V;
+  p.rc = rc;
+  p.nblk = nblk;
+  p.temperature = sp->temperature;
+  p.round = sp->round;
+  p.seed = sp->seed;
+  return lsp::launch_sample(p, dtype, static_cast<cudaStream_t>(stream));
+}

@@ -81,6 +81,9 @@ _f = {
                       POINTER(lsp_sample_params), c_void_p, c_void_p, c_void_p),
     "lsp_sample": _sig("lsp_sample", c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                        POINTER(lsp_sample_params), c_void_p, c_void_p, c_void_p),
+    "lsp_sample_noalloc": _sig("lsp_sample_noalloc", c_int, c_void_p, c_void_p, c_void_p, c_void_p,
+                               c_int, c_int, c_int, c_int, c_int, POINTER(lsp_sample_params),
+                               c_void_p, c_void_p, c_void_p, c_void_p),
     "lsp_linear_workspace_bytes": _sig("lsp_linear_workspace_bytes", c_size_t, c_int, c_int, c_int),
     "lsp_linear": _sig("lsp_linear", c_int, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                        c_int, c_void_p, c_size_t, c_void_p),
@@ -190,6 +193,15 @@ def lsp_sample(st, base_logits, prev_token, Ec, Wc, sp: lsp_sample_params, out_t
     _check(_f["lsp_sample"](st, _ptr(base_logits), _ptr(prev_token), _ptr(Ec), _ptr(Wc),
                             ctypes.byref(sp), _ptr(out_tokens), _ptr(out_logits), _stream(stream)),
            "lsp_sample")
+
+
+def lsp_sample_noalloc(base_logits, prev_token, Ec, Wc, dtype, C, B, V, rc,
+                       sp: lsp_sample_params, out_tokens, out_logits=None, dev_error=None,
+                       stream=None) -> None:
+    _check(_f["lsp_sample_noalloc"](_ptr(base_logits), _ptr(prev_token), _ptr(Ec), _ptr(Wc), dtype,
+                                    C, B, V, rc, ctypes.byref(sp), _ptr(out_tokens),
+                                    _ptr(out_logits), _ptr(dev_error), _stream(stream)),
+           "lsp_sample_noalloc")
 
 
 def lsp_linear_workspace_bytes(M: int, N: int, splits: int) -> int:
