@@ -243,10 +243,11 @@ int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, cons
 /* Dense projection Y = X W^T with the drafter's tensor-core GEMM (the kernel
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].
- *   M <= 512, K and N multiples of 16 bytes / element size.
- *   splits: split-K factor (1..16); workspace device bytes of at least
- *   lsp_linear_workspace_bytes(M, N, splits), zero-filled before its first use
- *   (the kernel leaves it reusable). */
+ *   M <= 512; K * element size a multiple of 16 bytes.
+ *   splits: split-K factor (1..16, at most the number of K blocks); with
+ *   splits > 1 the kernel writes fp32 partial sums to `workspace` (device, at
+ *   least lsp_linear_workspace_bytes(M, N, splits) bytes) and a second kernel
+ *   sums them in split order into Y. */
 size_t lsp_linear_workspace_bytes(int M, int N, int splits);
 int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype,
                int splits, void* workspace, size_t workspace_bytes, lsp_stream_t stream);

@@ -89,6 +89,8 @@ __global__ void __launch_bounds__(512)
   const int nthr = nwarps * 32;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = blockIdx.x / p.nkv, g = blockIdx.x % p.nkv;
+  griddep_launch();
+  griddep_wait();
   const int B = p.B, L = p.L, l = p.layer;
   const long long t = p.t[b];
   const int count = (int)(t < p.W ? t : p.W);
@@ -137,17 +139,19 @@ __global__ void __launch_bounds__(512)
     const int hh = hr / (16 - B), i = B + hr % (16 - B);
     *reinterpret_cast<uint4*>(sQ + (size_t)(hh * 16 + i) * row + c) = make_uint4(0, 0, 0, 0);
   }
-  // ---- block q (rep heads), k, v of KV head g: per-head RMSNorm + rotary for q, k
+  // ---- block q (rep heads), k, v of KV head g (sum of the projection's split-K
+  //      partials): per-head RMSNorm + rotary for q, k
   {
-    const bf16* qkv = static_cast<const bf16*>(p.qkv);
+    const float* qkv = p.qkv;
     const int ldq = (p.nq + 2 * p.nkv) * kHD;
+    const size_t pstride = (size_t)p.C * B * ldq;
     const bf16* qn = static_cast<const bf16*>(p.q_norm);
     const bf16* kn = static_cast<const bf16*>(p.k_norm);
     const int kinds = rep + 2;
     for (int item = warp; item < B * kinds; item += nwarps) {
       const int i = item / kinds, kind = item % kinds;
       const size_t mrow = (size_t)(b * B + i) * ldq;
-      const bf16* src;
+      const float* src;
       bf16* dst;
       if (kind < rep) {
         src = qkv + mrow + (size_t)(g * rep + kind) * kHD;
@@ -161,7 +165,11 @@ __global__ void __launch_bounds__(512)
       }
       float x[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) x[e] = to_f(src[lane + 32 * e]);
+      for (int e = 0; e < 4; ++e) {
+        float acc = src[lane + 32 * e];
+        for (int sp = 1; sp < p.qkv_splits; ++sp) acc += src[sp * pstride + lane + 32 * e];
+        x[e] = acc;
+      }
       if (kind <= rep) {
         const bf16* w = kind < rep ? qn : kn;
         const float ss = warp_sum(x[0] * x[0] + x[1] * x[1] + x[2] * x[2] + x[3] * x[3]);
@@ -316,26 +324,34 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
   float* sv = sk + B * d;
   float* ss = sv + B * d;                 // [B][ctx]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
-  const T* qkv = static_cast<const T*>(p.qkv);
+  griddep_launch();
+  griddep_wait();
+  const float* qkv = p.qkv;
   const int ldq = (p.nq + 2 * p.nkv) * d;
+  const size_t pstride = (size_t)p.C * B * ldq;
+  auto qkv_at = [&](const float* ptr, int e) {
+    float acc = ptr[e];
+    for (int sp = 1; sp < p.qkv_splits; ++sp) acc += ptr[sp * pstride + e];
+    return acc;
+  };
   for (int item = warp; item < 3 * B; item += nw) {
     const int i = item / 3, kind = item % 3;
     const size_t mrow = (size_t)(b * B + i) * ldq;
-    const T* src = qkv + mrow + (kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
-                                                                      : (size_t)(p.nq + p.nkv + g) * d);
+    const float* src = qkv + mrow + (kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
+                                                                          : (size_t)(p.nq + p.nkv + g) * d);
     float* dst = (kind == 0 ? sq : kind == 1 ? sk : sv) + i * d;
     if (kind == 2) {
-      for (int e = lane; e < d; e += 32) dst[e] = to_f(src[e]);
+      for (int e = lane; e < d; e += 32) dst[e] = qkv_at(src, e);
       continue;
     }
     float part = 0.f;
-    for (int e = lane; e < d; e += 32) part += to_f(src[e]) * to_f(src[e]);
+    for (int e = lane; e < d; e += 32) part += qkv_at(src, e) * qkv_at(src, e);
     const float rstd = rsqrtf(warp_sum(part) / (float)d + p.eps);
     const T* w = static_cast<const T*>(kind == 0 ? p.q_norm : p.k_norm);
     const float* cs = p.rope + (size_t)(b * B + i) * half * 2;
     for (int f = lane; f < half; f += 32) {
-      const float x1 = to_f(src[f]) * rstd * to_f(w[f]);
-      const float x2 = to_f(src[f + half]) * rstd * to_f(w[f + half]);
+      const float x1 = qkv_at(src, f) * rstd * to_f(w[f]);
+      const float x2 = qkv_at(src, f + half) * rstd * to_f(w[f + half]);
       dst[f] = x1 * cs[2 * f] - x2 * cs[2 * f + 1];
       dst[f + half] = x2 * cs[2 * f] + x1 * cs[2 * f + 1];
     }
@@ -418,7 +434,9 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
       cudaFuncSetAttribute(attn_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
       attr_set = true;
     }
-    attn_mma_kernel<<<p.C * p.nkv, a.nwarps * 32, a.bytes, s>>>(p, a.rep, ks, a.rows_bw);
+    if (launch_pdl(attn_mma_kernel, dim3(p.C * p.nkv), dim3(a.nwarps * 32), a.bytes, s, p, a.rep, ks,
+                   a.rows_bw) != cudaSuccess)
+      return LSP_ERR_CUDA;
   } else {
     const int ctx = p.B + p.W + p.R;
     const size_t smem = (size_t)(3 * p.B * p.d + p.B * ctx) * sizeof(float);
@@ -429,7 +447,8 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
                            227 * 1024);
       attr32 = true;
     }
-    attn_simple_kernel<float><<<p.C * p.nq, 128, smem, s>>>(p);
+    if (launch_pdl(attn_simple_kernel<float>, dim3(p.C * p.nq), dim3(128), smem, s, p) != cudaSuccess)
+      return LSP_ERR_CUDA;
   }
   return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }

@@ -6,18 +6,23 @@
 // large weight.  The kernel therefore puts 128 weight rows on the UMMA M axis
 // and the tokens on its N axis ("swap AB"): D^T[n][m] = sum_k W[n][k] X[m][k].
 //
-//   warp 0      TMA producer: one 128 x BK weight tile (16 KB) and the M x BK
-//               activation tile per stage into an S-deep mbarrier ring
+//   warp 0      TMA producer: `wt` 128 x BK weight tiles and the M x BK
+//               activation tile per stage into an S-deep mbarrier ring, plus
+//               L2 prefetches of the weight tiles `pd` stages ahead
 //   warp 1      TMEM allocation and the single-thread tcgen05.mma issue
-//   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulator, fused
-//               store / residual add / SwiGLU, or a split-K partial
+//   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulators and a fused
+//               store (fp32, storage dtype, SwiGLU) or a split-K partial
 //
-// Split-K partials go to a workspace; the last CTA of a tile (atomic ticket)
-// sums them in split order, so results are deterministic.  Every mbarrier wait
-// is bounded and records LSP_DEV_TIMEOUT instead of spinning forever.
+// Launched as a programmatic dependent: before the preceding kernel finishes,
+// the producer already streams this launch's weights (L2 prefetch and the
+// weight halves of the first stages); activation loads wait for it.  Split-K
+// partials are summed in split order by the consuming kernel, so results are
+// deterministic and no CTA waits on another.  Every mbarrier wait is bounded
+// and records LSP_DEV_TIMEOUT instead of spinning forever.
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <mutex>
 
 #include "common.cuh"
@@ -37,6 +42,8 @@ template <> struct GemmType<float> {
   static constexpr uint32_t FMT = 2;
 };
 
+constexpr uint32_t kTileBytes = kTileRows * 128;   // one weight tile per stage: 16 KB
+
 // Instruction descriptor: fp32 accumulate, A/B format `fmt`, both K-major,
 // N = n, M = 128.
 __device__ __forceinline__ uint32_t make_idesc(int n, uint32_t fmt) {
@@ -45,7 +52,7 @@ __device__ __forceinline__ uint32_t make_idesc(int n, uint32_t fmt) {
 }
 
 template <typename T>
-__device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int r, int m0,
+__device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int split, int r, int m0,
                                            const float* v, float* xchg) {
   const int M = p.M;
   if (p.mode == EPI_SWIGLU) {
@@ -75,13 +82,9 @@ __device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int r,
 #pragma unroll
     for (int j = 0; j < 16; ++j)
       if (m0 + j < M) Y[(size_t)(m0 + j) * p.ldy + n] = from_f<T>(v[j]);
-  } else if (p.mode == EPI_RESID) {
-    float* Y = static_cast<float*>(p.Y);
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (m0 + j < M) Y[(size_t)(m0 + j) * p.ldy + n] += v[j];
   } else {
     float* Y = static_cast<float*>(p.Y);
+    if (p.mode == EPI_PARTIAL) Y += (size_t)split * M * p.ldy;
 #pragma unroll
     for (int j = 0; j < 16; ++j)
       if (m0 + j < M) Y[(size_t)(m0 + j) * p.ldy + n] = v[j];
@@ -98,19 +101,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int S = p.stages;
-  const uint32_t stage_a = kTileRows * 128;
+  const uint32_t stage_a = (uint32_t)p.wt * kTileBytes;
   const uint32_t stage_bytes = stage_a + (uint32_t)p.m_pad * 128;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 1);
-  volatile int* s_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);  // [0] last CTA, [1] abort
+  volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int tile = blockIdx.x;
+  const int tile0 = blockIdx.x * p.wt;
+  const int ntl = min(p.wt, p.n_tiles - tile0);                // weight tiles of this CTA
   const int split = blockIdx.y;
   const int kb0 = (int)((long long)split * p.kblocks / p.splits);
   const int kb1 = (int)((long long)(split + 1) * p.kblocks / p.splits);
   const int nk = kb1 - kb0;
+  const uint32_t expect = (uint32_t)ntl * kTileBytes + (uint32_t)p.m_pad * 128;
 
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -123,8 +128,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(acc_bar, 1);
-    s_flag[0] = 0;
-    s_flag[1] = 0;
+    *s_abort = 0;
     fence_barrier_init();
     tma_prefetch_desc(&ta0);
     tma_prefetch_desc(&tb);
@@ -133,6 +137,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  griddep_launch();
   const uint32_t tmem_base = *tmem_slot;
 
   int issued = 0;
@@ -140,29 +145,70 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ------------------------------------------------------------ TMA producer
     const uint64_t pol_w = policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
-    int seg = 0;
-    if (p.mode != EPI_SWIGLU) {
+    // weight tile w of this CTA: tensor map and first row
+    auto a_src = [&](int w, const CUtensorMap** ta, int* row) {
+      const int tile = tile0 + w;
+      int seg = 0;
       if (p.nseg > 2 && tile >= p.seg_tile0[2]) seg = 2;
       else if (p.nseg > 1 && tile >= p.seg_tile0[1]) seg = 1;
+      *ta = seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2);
+      *row = (tile - p.seg_tile0[seg]) * kTileRows;
+    };
+    auto load_a = [&](int i, uint32_t sa, uint32_t bar) {
+      const int kx = (kb0 + i) * G::BK;
+      for (int w = 0; w < ntl; ++w) {
+        if (p.mode == EPI_SWIGLU) {
+          const int row = (tile0 + w) * 64;
+          tma_load_2d(sa + w * kTileBytes, &ta0, bar, kx, row, pol_w);
+          tma_load_2d(sa + w * kTileBytes + 64 * 128, &ta1, bar, kx, row, pol_w);
+        } else {
+          const CUtensorMap* ta;
+          int row;
+          a_src(w, &ta, &row);
+          tma_load_2d(sa + w * kTileBytes, ta, bar, kx, row, pol_w);
+        }
+      }
+    };
+    auto prefetch_a = [&](int i) {
+      const int kx = (kb0 + i) * G::BK;
+      for (int w = 0; w < ntl; ++w) {
+        if (p.mode == EPI_SWIGLU) {
+          tma_prefetch_l2(&ta0, kx, (tile0 + w) * 64);
+          tma_prefetch_l2(&ta1, kx, (tile0 + w) * 64);
+        } else {
+          const CUtensorMap* ta;
+          int row;
+          a_src(w, &ta, &row);
+          tma_prefetch_l2(ta, kx, row);
+        }
+      }
+    };
+    auto load_b = [&](int i, uint32_t sb, uint32_t bar) {
+      const int kx = (kb0 + i) * G::BK;
+      for (int tt = 0; tt < p.n_tok_tiles; ++tt)
+        tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, bar, kx, tt * p.bn, pol_x);
+    };
+    // Weights do not depend on the preceding kernel: start streaming them now.
+    int next_pf = 0;
+    const int pre = min(S, nk);
+    while (next_pf < min(p.pd, nk)) prefetch_a(next_pf++);
+    for (int i = 0; i < pre; ++i) {
+      mbar_expect_tx(full_bar(i), expect);
+      load_a(i, smem_u32(smem + (size_t)i * stage_bytes), full_bar(i));
     }
-    const CUtensorMap* ta = seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2);
-    const int arow = (tile - p.seg_tile0[seg]) * kTileRows;
-    for (int i = 0; i < nk; ++i) {
+    griddep_wait();                       // activations come from the preceding kernel
+    for (int i = 0; i < pre; ++i)
+      load_b(i, smem_u32(smem + (size_t)i * stage_bytes) + stage_a, full_bar(i));
+    issued = pre;
+    for (int i = pre; i < nk; ++i) {
+      while (next_pf < nk && next_pf < i + p.pd) prefetch_a(next_pf++);
       const int s = i % S;
       const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(empty_bar(s), ph ^ 1u, p.err)) { s_flag[1] = 1; break; }
-      mbar_expect_tx(full_bar(s), stage_bytes);
+      if (!mbar_wait(empty_bar(s), ph ^ 1u, p.err)) { *s_abort = 1; break; }
+      mbar_expect_tx(full_bar(s), expect);
       const uint32_t sa = smem_u32(smem + (size_t)s * stage_bytes);
-      const uint32_t sb = sa + stage_a;
-      const int kx = (kb0 + i) * G::BK;
-      if (p.mode == EPI_SWIGLU) {
-        tma_load_2d(sa, &ta0, full_bar(s), kx, tile * 64, pol_w);
-        tma_load_2d(sa + 64 * 128, &ta1, full_bar(s), kx, tile * 64, pol_w);
-      } else {
-        tma_load_2d(sa, ta, full_bar(s), kx, arow, pol_w);
-      }
-      for (int tt = 0; tt < p.n_tok_tiles; ++tt)
-        tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, full_bar(s), kx, tt * p.bn, pol_x);
+      load_a(i, sa, full_bar(s));
+      load_b(i, sa + stage_a, full_bar(s));
       issued = i + 1;
     }
   } else if (warp == 1 && lane == 0) {
@@ -171,20 +217,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     for (int i = 0; i < nk; ++i) {
       const int s = i % S;
       const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(full_bar(s), ph, p.err)) { s_flag[1] = 1; break; }
+      if (!mbar_wait(full_bar(s), ph, p.err)) { *s_abort = 1; break; }
       tc_fence_after();
       const uint32_t sa = smem_u32(smem + (size_t)s * stage_bytes);
       const uint32_t sb = sa + stage_a;
 #pragma unroll
       for (int kk = 0; kk < G::BK / G::UK; ++kk) {
-        const uint64_t ad = sdesc_sw128(sa + kk * 32);
-        for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
-          const uint64_t bd = sdesc_sw128(sb + (uint32_t)(tt * p.bn * 128) + kk * 32);
-          const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-          if constexpr (sizeof(T) == 2)
-            umma_f16(tmem_base + (uint32_t)(tt * p.bn), ad, bd, idesc, acc);
-          else
-            umma_tf32(tmem_base + (uint32_t)(tt * p.bn), ad, bd, idesc, acc);
+        for (int w = 0; w < ntl; ++w) {
+          const uint64_t ad = sdesc_sw128(sa + w * kTileBytes + kk * 32);
+          for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
+            const uint64_t bd = sdesc_sw128(sb + (uint32_t)(tt * p.bn * 128) + kk * 32);
+            const uint32_t col = (uint32_t)((w * p.n_tok_tiles + tt) * p.bn);
+            const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+            if constexpr (sizeof(T) == 2)
+              umma_f16(tmem_base + col, ad, bd, idesc, acc);
+            else
+              umma_tf32(tmem_base + col, ad, bd, idesc, acc);
+          }
         }
       }
       umma_commit(empty_bar(s));
@@ -194,62 +243,27 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;
     const int r = q * 32 + lane;
-    const int etid = threadIdx.x - 64;
     float* xchg = reinterpret_cast<float*>(smem);   // pipeline smem is idle once acc_bar fired
+    griddep_wait();
     const bool ok = mbar_wait(acc_bar, 0, p.err);
-    if (!ok) s_flag[1] = 1;
+    if (!ok) *s_abort = 1;
     tc_fence_after();
     named_bar(1, 128);
-    const bool abort = s_flag[1] != 0;
-    const uint32_t tb_addr = tmem_base + ((uint32_t)(q * 32) << 16);
-    if (!abort) {
-      if (p.splits == 1) {
+    if (*s_abort == 0) {
+      const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
+      for (int w = 0; w < ntl; ++w)
         for (int tt = 0; tt < p.n_tok_tiles; ++tt)
           for (int c0 = 0; c0 < p.bn; c0 += 16) {
             float v[16];
-            tmem_ld16(tb_addr + (uint32_t)(tt * p.bn + c0), v);
-            emit_chunk<T>(p, tile, r, tt * p.bn + c0, v, xchg);
+            tmem_ld16(lane_base + (uint32_t)((w * p.n_tok_tiles + tt) * p.bn + c0), v);
+            emit_chunk<T>(p, tile0 + w, split, r, tt * p.bn + c0, v, xchg);
           }
-      } else {
-        float* part = p.ws + (size_t)(tile * p.splits + split) * p.m_pad * kTileRows;
-        for (int tt = 0; tt < p.n_tok_tiles; ++tt)
-          for (int c0 = 0; c0 < p.bn; c0 += 16) {
-            float v[16];
-            tmem_ld16(tb_addr + (uint32_t)(tt * p.bn + c0), v);
-            const int m0 = tt * p.bn + c0;
-#pragma unroll
-            for (int j = 0; j < 16; ++j) part[(size_t)(m0 + j) * kTileRows + r] = v[j];
-          }
-        __threadfence();
-        named_bar(1, 128);
-        if (etid == 0) {
-          const int old = atomicAdd(&p.counters[tile], 1);
-          s_flag[0] = (old == p.splits - 1) ? 1 : 0;
-        }
-        named_bar(1, 128);
-        if (s_flag[0]) {
-          __threadfence();
-          const float* base = p.ws + (size_t)tile * p.splits * p.m_pad * kTileRows;
-          for (int m0 = 0; m0 < p.M; m0 += 16) {
-            float v[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] = 0.0f;
-            for (int s2 = 0; s2 < p.splits; ++s2) {
-              const float* ps = base + (size_t)s2 * p.m_pad * kTileRows;
-#pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] += __ldcg(ps + (size_t)(m0 + j) * kTileRows + r);
-            }
-            emit_chunk<T>(p, tile, r, m0, v, xchg);
-          }
-          if (etid == 0) p.counters[tile] = 0;
-        }
-      }
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 0 && lane == 0 && s_flag[1]) {
+  if (warp == 0 && lane == 0 && *s_abort) {
     // A wait gave up: let every TMA copy this CTA issued land before exit.
     for (int i = (issued > S ? issued - S : 0); i < issued; ++i)
       mbar_wait(full_bar(i % S), (uint32_t)(i / S) & 1u, p.err);
@@ -257,6 +271,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, (uint32_t)p.tmem_cols);
+  }
+}
+
+__global__ void sum_partials_kernel(const float* __restrict__ part, int splits, size_t n,
+                                    float* __restrict__ y) {
+  griddep_launch();
+  griddep_wait();
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x) {
+    float acc = part[i];
+    for (int s = 1; s < splits; ++s) acc += part[(size_t)s * n + i];
+    y[i] = acc;
   }
 }
 
@@ -302,38 +328,65 @@ int gemm_tiles(int mode, const int* seg_rows, int nseg) {
   return t;
 }
 
+int gemm_kblocks(int K, int dtype) {
+  const int bk = dtype == LSP_DTYPE_BF16 ? 64 : 32;
+  return (K + bk - 1) / bk;
+}
+
 static void token_tiling(int M, int* bn, int* ntt) {
   *ntt = (M + 255) / 256;
   int per = (M + *ntt - 1) / *ntt;
   *bn = std::max(16, (per + 15) / 16 * 16);
 }
 
-size_t gemm_ws_bytes(int M, int n_tiles, int splits) {
-  int bn, ntt;
-  token_tiling(M, &bn, &ntt);
-  return splits <= 1 ? 0 : (size_t)n_tiles * splits * (size_t)bn * ntt * kTileRows * sizeof(float);
-}
-
 static constexpr int kSmemBudget = 227 * 1024;
 
+// Tuning overrides for measurement sweeps: LSP_GEMM_WT (weight tiles per CTA),
+// LSP_GEMM_PD (L2 prefetch distance in k-blocks), LSP_GEMM_STAGES.  Unset or
+// non-positive values keep the defaults; the values never change results.
+static int tuning(const char* name) {
+  const char* v = std::getenv(name);
+  return v ? std::atoi(v) : 0;
+}
+
+double gemm_partial_cost(int M) {
+  int bn, ntt;
+  token_tiling(M, &bn, &ntt);
+  return (double)(bn * ntt) / 64.0;
+}
+
 // split-K factor: minimise waves x (k-blocks per CTA + fixed per-CTA overhead)
-int gemm_auto_splits(int n_tiles, int kblocks, int num_sms) {
+// (partial_cost: the per-CTA cost of writing and re-reading one fp32 partial,
+// in k-block units)
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost) {
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(16, kblocks); ++s) {
-    const long long ctas = (long long)n_tiles * s;
+    const long long ctas = (long long)n_ctas * s;
     const long long waves = (ctas + num_sms - 1) / num_sms;
-    const double per = (double)((kblocks + s - 1) / s) + 3.0 + (s > 1 ? 1.5 : 0.0);
+    const double per = (double)((kblocks + s - 1) / s) + 4.0 + (s > 1 ? partial_cost : 0.0);
     const double cost = (double)waves * per;
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
   return splits;
 }
 
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt) {
+  int bn, ntt;
+  token_tiling(M, &bn, &ntt);
+  const int m_pad = bn * ntt;
+  // one weight tile per CTA: two tiles sharing the activation tile measured slower
+  if (*wt <= 0) *wt = 1;
+  const int kblocks = gemm_kblocks(K, dtype);
+  const int n_ctas = (n_tiles + *wt - 1) / *wt;
+  if (*splits <= 0)
+    *splits = mode == EPI_PARTIAL ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M)) : 1;
+  *splits = std::max(1, std::min(*splits, kblocks));
+}
+
 int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
-              const int* seg_rows, int nseg, int mode, void* Y, int ldy, float* ws,
-              size_t ws_bytes, int* counters, int n_counters, unsigned* err, int num_sms,
-              int splits) {
+              const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
+              int num_sms, int splits, int wt) {
   if (M < 1 || M > 512 || K < 1 || nseg < 1 || nseg > 3) return LSP_ERR_SHAPE;
   if (mode == EPI_SWIGLU && nseg != 2) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
@@ -350,7 +403,6 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   p.N = 0;
   if (mode == EPI_SWIGLU) {
     p.N = seg_rows[0];
-    p.seg_tile0[0] = p.seg_tile0[1] = p.seg_tile0[2] = 0;
   } else {
     int t0 = 0;
     for (int i = 0; i < 3; ++i) {
@@ -359,27 +411,32 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     }
     for (int i = 0; i < nseg; ++i) p.N += seg_rows[i];
   }
-  const int bk = 128 / es;
-  p.kblocks = (K + bk - 1) / bk;
+  p.kblocks = gemm_kblocks(K, dtype);
   token_tiling(M, &p.bn, &p.n_tok_tiles);
   p.m_pad = p.bn * p.n_tok_tiles;
+  if (wt <= 0 && tuning("LSP_GEMM_WT") > 0) wt = tuning("LSP_GEMM_WT");
+  gemm_choose(dtype, M, K, p.n_tiles, mode, num_sms, &splits, &wt);
+  if (wt < 1 || wt > 2 || wt * p.m_pad > 512) return LSP_ERR_SHAPE;
+  p.wt = wt;
   int cols = 32;
-  while (cols < p.m_pad) cols *= 2;
+  while (cols < wt * p.m_pad) cols *= 2;
   p.tmem_cols = cols;
-  const int stage_bytes = kTileRows * 128 + p.m_pad * 128;
+  const int stage_bytes = wt * (int)kTileBytes + p.m_pad * 128;
   p.stages = std::min(8, (kSmemBudget - 2048) / stage_bytes);
+  const int n_ctas = (p.n_tiles + wt - 1) / wt;
+  // With CTAs to spare, two 2-stage CTAs per SM beat one deep CTA: one CTA's
+  // prologue and epilogue overlap the other's weight stream (same bytes in flight).
+  if ((long long)n_ctas * splits >= (long long)num_sms * 5 / 4 && 2 * stage_bytes + 2048 <= kSmemBudget / 2 &&
+      2 * wt * p.m_pad <= 512)
+    p.stages = 2;
+  if (tuning("LSP_GEMM_STAGES") > 0) p.stages = std::min(p.stages, tuning("LSP_GEMM_STAGES"));
   if (p.stages < 2) return LSP_ERR_SHAPE;
-  if (splits <= 0) splits = gemm_auto_splits(p.n_tiles, p.kblocks, num_sms);
-  splits = std::max(1, std::min(splits, p.kblocks));
-  if (splits > 1) {
-    if (!ws || !counters || n_counters < p.n_tiles || gemm_ws_bytes(M, p.n_tiles, splits) > ws_bytes)
-      return LSP_ERR_SHAPE;
-  }
+  p.pd = 0;                             // weight k-blocks prefetched into L2 ahead (off: it re-read DRAM)
+  if (std::getenv("LSP_GEMM_PD")) p.pd = std::max(0, tuning("LSP_GEMM_PD"));
+  if (splits > 1 && mode != EPI_PARTIAL) return LSP_ERR_SHAPE;
   p.splits = splits;
   p.Y = Y;
   p.ldy = ldy;
-  p.ws = ws;
-  p.counters = counters;
   p.err = err;
   op->dtype = dtype;
   const int box_rows = mode == EPI_SWIGLU ? 64 : kTileRows;
@@ -389,7 +446,7 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     if ((rc = make_map(&op->a[i], dtype, W[si], K, seg_rows[si], box_rows)) != LSP_OK) return rc;
   }
   if ((rc = make_map(&op->b, dtype, X, K, M, p.bn)) != LSP_OK) return rc;
-  op->grid = dim3((unsigned)p.n_tiles, (unsigned)splits, 1);
+  op->grid = dim3((unsigned)n_ctas, (unsigned)splits, 1);
   op->smem = (size_t)p.stages * stage_bytes + 1024 + 256;
   return LSP_OK;
 }
@@ -400,13 +457,21 @@ static int launch_t(const GemmOp* op, cudaStream_t s) {
   std::call_once(once, [] {
     cudaFuncSetAttribute(gemm_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
   });
-  gemm_kernel<T><<<op->grid, kGemmThreads, op->smem, s>>>(op->a[0], op->a[1], op->a[2], op->b,
-                                                           op->p);
-  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+  const cudaError_t e = launch_pdl(gemm_kernel<T>, op->grid, dim3(kGemmThreads), op->smem, s,
+                                   op->a[0], op->a[1], op->a[2], op->b, op->p);
+  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 int gemm_launch(const GemmOp* op, cudaStream_t s) {
   return op->dtype == LSP_DTYPE_BF16 ? launch_t<bf16>(op, s) : launch_t<float>(op, s);
+}
+
+int launch_sum_partials(const float* part, int splits, size_t n, float* y, cudaStream_t s) {
+  const unsigned blocks = (unsigned)std::min<size_t>((n + 255) / 256, 4096);
+  return launch_pdl(sum_partials_kernel, dim3(blocks), dim3(256), 0, s, part, splits, n, y) ==
+                 cudaSuccess
+             ? LSP_OK
+             : LSP_ERR_CUDA;
 }
 
 }  // namespace lsp

@@ -88,6 +88,8 @@ __global__ void __launch_bounds__(kSampThreads) sample_step_kernel(const SampleP
   T* e_s = reinterpret_cast<T*>(corr_s + kSampWarps * kMaxC * 17);        // [C8][lde]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  griddep_launch();
+  griddep_wait();
 
   // ---- y_{i-1} for every request
   if (step == 0) {
@@ -223,6 +225,8 @@ __global__ void __launch_bounds__(kSampThreads) sample_step_kernel(const SampleP
 
 __global__ void __launch_bounds__(kSampThreads) sample_final_kernel(const SampleParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  griddep_launch();
+  griddep_wait();
   for (int b = warp; b < p.C; b += kSampWarps) {
     const int y = resolve_prev(p, (p.B - 1) & 1, b, lane);
     if (lane == 0) p.out_tokens[(size_t)b * p.B + p.B - 1] = y;
@@ -258,13 +262,14 @@ int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
     attr_set = true;
   }
   for (int step = 0; step < p.B; ++step) {
-    if (dtype == LSP_DTYPE_BF16)
-      sample_step_kernel<bf16><<<p.nblk, kSampThreads, smem, s>>>(p, step);
-    else
-      sample_step_kernel<float><<<p.nblk, kSampThreads, smem, s>>>(p, step);
+    cudaError_t e = dtype == LSP_DTYPE_BF16
+                        ? launch_pdl(sample_step_kernel<bf16>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step)
+                        : launch_pdl(sample_step_kernel<float>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step);
+    if (e != cudaSuccess) return LSP_ERR_CUDA;
   }
-  sample_final_kernel<<<1, kSampThreads, 0, s>>>(p);
-  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+  if (launch_pdl(sample_final_kernel, dim3(1), dim3(kSampThreads), 0, s, p) != cudaSuccess)
+    return LSP_ERR_CUDA;
+  return LSP_OK;
 }
 
 int launch_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint32_t* out,

@@ -1,14 +1,17 @@
 // Small fused row ops of the drafter forward.
 //
-// combine_kernel (Sec. 2.3, input slots): x_i = E[u_i] + P_i + c_t with u_0 = a
-// (the committed token) and the mask embedding for slots holding -1, written
-// to the fp32 residual stream, fused with the first layer's input RMSNorm; the
-// same launch fills the rotary cos/sin table of every (request, slot) at
-// absolute position t + i, with the angle formed and reduced in fp64 so that
-// positions near 1.3e5 keep full fp32 accuracy.
+// combine_kernel (Sec. 2.3, input slots): c_t is the sum of the boundary-fusion
+// GEMM's split-K partials; x_i = E[u_i] + P_i + c_t with u_0 = a (the committed
+// token) and the mask embedding for slots holding -1, written to the fp32
+// residual stream and fused with the first layer's input RMSNorm.  The same
+// launch fills the rotary cos/sin table of every (request, slot) at absolute
+// position t + i: the angle is formed and reduced modulo 2*pi in fp64, so
+// positions near 1.3e5 keep full fp32 accuracy, and sin/cos run in fp32.
 //
-// rmsnorm_kernel: x / sqrt(mean(x^2) + eps) * w (Qwen3 RMSNorm) of fp32 rows
-// into the storage dtype that the next projection's TMA reads.
+// resid_norm_kernel: x += sum of a projection's split-K partials (the
+// residual add of the o and down projections, in split order), then
+// x / sqrt(mean(x^2) + eps) * w (Qwen3 RMSNorm) into the storage dtype that
+// the next projection's TMA reads.
 #include "common.cuh"
 #include "lsp_internal.h"
 
@@ -37,24 +40,32 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParams p) {
   __shared__ float red[32];
+  __shared__ double inv_freq[128];
+  griddep_launch();
   const int M = p.C * p.B;
   if ((int)blockIdx.x >= M) {
     // rotary table of request b: rope[b][i][f] = (cos, sin)(pos * theta^(-2f/d))
     const int b = blockIdx.x - M;
     const int half = p.d / 2;
+    for (int f = threadIdx.x; f < half; f += blockDim.x)
+      inv_freq[f] = pow(p.theta, -2.0 * (double)f / (double)p.d);
+    __syncthreads();
+    griddep_wait();
     const long long t0 = p.t[b];
+    const double two_pi = 6.283185307179586476925286766559;
     for (int idx = threadIdx.x; idx < p.B * half; idx += blockDim.x) {
       const int i = idx / half, f = idx % half;
-      const double inv = pow(p.theta, -2.0 * (double)f / (double)p.d);
-      const double ang = (double)(t0 + i) * inv;
-      double sn, cs;
-      sincos(ang, &sn, &cs);
+      const double ang = (double)(t0 + i) * inv_freq[f];
+      const double red_ang = ang - rint(ang * (1.0 / two_pi)) * two_pi;
+      float sn, cs;
+      sincosf((float)red_ang, &sn, &cs);
       float* dst = p.rope + ((size_t)(b * p.B + i) * half + f) * 2;
-      dst[0] = (float)cs;
-      dst[1] = (float)sn;
+      dst[0] = cs;
+      dst[1] = sn;
     }
     return;
   }
+  griddep_wait();
   const int m = blockIdx.x, b = m / p.B, i = m % p.B;
   int u = p.tokens[(size_t)b * p.B + i];
   const bool ok = (i == 0) ? (u >= 0 && u < p.V) : (u >= -1 && u < p.V);
@@ -65,6 +76,7 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   const T* src = u >= 0 ? static_cast<const T*>(p.embed) + (size_t)u * p.H
                         : static_cast<const T*>(p.mask_emb);
   const T* pos = static_cast<const T*>(p.pos) + (size_t)i * p.H;
+  const size_t cstride = (size_t)p.C * p.H;
   const float* c = p.c + (size_t)b * p.H;
   float xv[kMaxPerThread];
   float ss = 0.f;
@@ -73,7 +85,9 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
     const int h = threadIdx.x + k * kRowThreads;
     xv[k] = 0.f;
     if (h < p.H) {
-      xv[k] = to_f(src[h]) + to_f(pos[h]) + c[h];
+      float cv = c[h];
+      for (int s = 1; s < p.c_splits; ++s) cv += c[s * cstride + h];
+      xv[k] = to_f(src[h]) + to_f(pos[h]) + cv;
       p.x[(size_t)m * p.H + h] = xv[k];
       ss += xv[k] * xv[k];
     }
@@ -90,18 +104,27 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
 
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads)
-    rmsnorm_kernel(const float* __restrict__ x, const T* __restrict__ w, T* __restrict__ out, int H,
-                   float eps) {
+    resid_norm_kernel(float* __restrict__ x, const float* __restrict__ part, int splits,
+                      const T* __restrict__ w, T* __restrict__ out, int M, int H, float eps) {
   __shared__ float red[32];
+  griddep_launch();
+  griddep_wait();
   const int m = blockIdx.x;
-  const float* row = x + (size_t)m * H;
+  float* row = x + (size_t)m * H;
+  const size_t pstride = (size_t)M * H;
   float xv[kMaxPerThread];
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < kMaxPerThread; ++k) {
     const int h = threadIdx.x + k * kRowThreads;
-    xv[k] = h < H ? row[h] : 0.f;
-    ss += xv[k] * xv[k];
+    xv[k] = 0.f;
+    if (h < H) {
+      float v = row[h];
+      for (int s = 0; s < splits; ++s) v += part[s * pstride + (size_t)m * H + h];
+      xv[k] = v;
+      if (splits > 0) row[h] = v;
+      ss += v * v;
+    }
   }
   const float rstd = rsqrtf(block_sum(ss, red) / (float)H + eps);
 #pragma unroll
@@ -112,25 +135,25 @@ __global__ void __launch_bounds__(kRowThreads)
 }
 
 int launch_combine(const CombineParams& p, int dtype, cudaStream_t s) {
-  if (p.H > kRowThreads * kMaxPerThread) return LSP_ERR_SHAPE;
+  if (p.H > kRowThreads * kMaxPerThread || p.d / 2 > 128) return LSP_ERR_SHAPE;
   const dim3 grid(p.C * p.B + p.C);
-  if (dtype == LSP_DTYPE_BF16)
-    combine_kernel<bf16><<<grid, kRowThreads, 0, s>>>(p);
-  else
-    combine_kernel<float><<<grid, kRowThreads, 0, s>>>(p);
-  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+  cudaError_t e = dtype == LSP_DTYPE_BF16
+                      ? launch_pdl(combine_kernel<bf16>, grid, dim3(kRowThreads), 0, s, p)
+                      : launch_pdl(combine_kernel<float>, grid, dim3(kRowThreads), 0, s, p);
+  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
-int launch_rmsnorm(const float* x, const void* w, void* out, int M, int H, float eps, int dtype,
-                   cudaStream_t s) {
+int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
+                      int H, float eps, int dtype, cudaStream_t s) {
   if (H > kRowThreads * kMaxPerThread) return LSP_ERR_SHAPE;
+  cudaError_t e;
   if (dtype == LSP_DTYPE_BF16)
-    rmsnorm_kernel<bf16><<<M, kRowThreads, 0, s>>>(x, static_cast<const bf16*>(w),
-                                                   static_cast<bf16*>(out), H, eps);
+    e = launch_pdl(resid_norm_kernel<bf16>, dim3(M), dim3(kRowThreads), 0, s, x, part, splits,
+                   static_cast<const bf16*>(w), static_cast<bf16*>(out), M, H, eps);
   else
-    rmsnorm_kernel<float><<<M, kRowThreads, 0, s>>>(x, static_cast<const float*>(w),
-                                                    static_cast<float*>(out), H, eps);
-  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+    e = launch_pdl(resid_norm_kernel<float>, dim3(M), dim3(kRowThreads), 0, s, x, part, splits,
+                   static_cast<const float*>(w), static_cast<float*>(out), M, H, eps);
+  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 }  // namespace lsp

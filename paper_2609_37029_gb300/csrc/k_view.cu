@@ -39,6 +39,8 @@ __global__ void __launch_bounds__(kViewThreads)
   const int rep = p.nq / p.nkv;
   const int Q = rep * p.R;                      // queries handled by this CTA
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  griddep_launch();
+  griddep_wait();
 
   int delta = p.acc[b];
   if (delta < 0 || delta > p.rows) {
@@ -183,15 +185,16 @@ static int launch_dpl(const ViewParams& p, cudaStream_t s) {
   const int qpw = (Q + kViewWarps - 1) / kViewWarps;
   const size_t smem = 2 * kViewChunk * DPL * 32 * sizeof(float);
   const dim3 grid(p.C * p.L * p.nkv);
+  cudaError_t e;
   if (qpw <= 4)
-    view_update_kernel<T, DPL, 4><<<grid, kViewThreads, smem, s>>>(p);
+    e = launch_pdl(view_update_kernel<T, DPL, 4>, grid, dim3(kViewThreads), smem, s, p);
   else if (qpw <= 8)
-    view_update_kernel<T, DPL, 8><<<grid, kViewThreads, smem, s>>>(p);
+    e = launch_pdl(view_update_kernel<T, DPL, 8>, grid, dim3(kViewThreads), smem, s, p);
   else if (qpw <= 16)
-    view_update_kernel<T, DPL, 16><<<grid, kViewThreads, smem, s>>>(p);
+    e = launch_pdl(view_update_kernel<T, DPL, 16>, grid, dim3(kViewThreads), smem, s, p);
   else
     return LSP_ERR_SHAPE;
-  return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 int launch_view_update(const ViewParams& p, int dtype, cudaStream_t s) {

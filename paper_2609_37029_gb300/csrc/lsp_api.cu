@@ -65,11 +65,9 @@ struct lsp_state {
   int* done = nullptr;
   // workspace
   void* ws = nullptr;
-  float *c = nullptr, *x = nullptr, *logits = nullptr, *rope = nullptr, *gemm_ws = nullptr;
-  void *xn = nullptr, *qkv = nullptr, *o = nullptr, *act = nullptr;
-  int* gemm_cnt = nullptr;
-  size_t gemm_ws_bytes = 0;
-  int gemm_cnt_n = 0;
+  float *x = nullptr, *logits = nullptr, *rope = nullptr, *part = nullptr;
+  void *xn = nullptr, *o = nullptr, *act = nullptr;
+  size_t part_bytes = 0;
   float* part_val = nullptr;
   int* part_idx = nullptr;
   int nblk = 0;
@@ -148,16 +146,15 @@ static void free_state(lsp_state* st) {
   delete st;
 }
 
-// Projection shapes of one round, for sizing the split-K workspace.
-static void projection_shapes(const lsp_config& c, int* M, int* K, int* rows0, int* mode, int* n) {
+// Projections that write split-K partials (summed by their consumer): their
+// token rows, reduction length and output features, for sizing the buffer.
+static void partial_shapes(const lsp_config& c, int* M, int* K, int* N, int* n) {
   const int Mt = c.C * c.B;
   int i = 0;
-  M[i] = c.C; K[i] = c.L * c.H; rows0[i] = c.H; mode[i++] = EPI_F32;                 // fusion
-  M[i] = Mt; K[i] = c.H; rows0[i] = (c.nq + 2 * c.nkv) * c.d; mode[i++] = EPI_T;     // q|k|v
-  M[i] = Mt; K[i] = c.nq * c.d; rows0[i] = c.H; mode[i++] = EPI_RESID;               // o
-  M[i] = Mt; K[i] = c.H; rows0[i] = c.F; mode[i++] = EPI_SWIGLU;                     // gate|up
-  M[i] = Mt; K[i] = c.F; rows0[i] = c.H; mode[i++] = EPI_RESID;                      // down
-  M[i] = Mt; K[i] = c.H; rows0[i] = c.V; mode[i++] = EPI_F32;                        // LM head
+  M[i] = c.C; K[i] = c.L * c.H; N[i++] = c.H;                      // boundary fusion
+  M[i] = Mt; K[i] = c.H; N[i++] = (c.nq + 2 * c.nkv) * c.d;        // q | k | v
+  M[i] = Mt; K[i] = c.nq * c.d; N[i++] = c.H;                      // o
+  M[i] = Mt; K[i] = c.F; N[i++] = c.H;                             // down
   *n = i;
 }
 
@@ -203,44 +200,37 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   // ---- workspace
   const size_t es = esize(c.dtype);
   const int M = c.C * c.B;
-  int pm[8], pk[8], prow[8], pmode[8], np;
-  projection_shapes(c, pm, pk, prow, pmode, &np);
-  size_t gws = 0;
-  int gcnt = 0;
+  int pm[8], pk[8], pn[8], np;
+  partial_shapes(c, pm, pk, pn, &np);
+  size_t pbytes = 0;
   for (int i = 0; i < np; ++i) {
-    const int tiles = gemm_tiles(pmode[i], prow + i, 1);
-    gcnt = std::max(gcnt, tiles);
-    const int kblocks = (pk[i] * (int)es + 127) / 128;
-    gws = std::max(gws, gemm_ws_bytes(pm[i], tiles, gemm_auto_splits(tiles, kblocks, st->num_sms)));
+    int splits = 0, wt = 0;
+    const int rows[1] = {pn[i]};
+    gemm_choose(c.dtype, pm[i], pk[i], gemm_tiles(EPI_PARTIAL, rows, 1), EPI_PARTIAL, st->num_sms,
+                &splits, &wt);
+    pbytes = std::max(pbytes, (size_t)splits * pm[i] * pn[i] * sizeof(float));
   }
   st->nblk = sample_blocks(st->num_sms);
   off = 0;
-  const size_t w_c = off; off = align256(off + (size_t)c.C * c.H * 4);
   const size_t w_x = off; off = align256(off + (size_t)M * c.H * 4);
   const size_t w_xn = off; off = align256(off + (size_t)M * c.H * es);
-  const size_t w_qkv = off; off = align256(off + (size_t)M * (c.nq + 2 * c.nkv) * c.d * es);
   const size_t w_o = off; off = align256(off + (size_t)M * c.nq * c.d * es);
   const size_t w_act = off; off = align256(off + (size_t)M * c.F * es);
   const size_t w_log = off; off = align256(off + (size_t)M * c.V * 4);
   const size_t w_rope = off; off = align256(off + (size_t)M * (c.d / 2) * 2 * 4);
-  const size_t w_gws = off; off = align256(off + gws);
-  const size_t w_gcnt = off; off = align256(off + (size_t)gcnt * 4);
+  const size_t w_part = off; off = align256(off + pbytes);
   const size_t w_pv = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
   const size_t w_pi = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
   if (cudaMalloc(&st->ws, off) != cudaSuccess) { free_state(st); return LSP_ERR_NOMEM; }
   char* w = static_cast<char*>(st->ws);
-  st->c = reinterpret_cast<float*>(w + w_c);
   st->x = reinterpret_cast<float*>(w + w_x);
   st->xn = w + w_xn;
-  st->qkv = w + w_qkv;
   st->o = w + w_o;
   st->act = w + w_act;
   st->logits = reinterpret_cast<float*>(w + w_log);
   st->rope = reinterpret_cast<float*>(w + w_rope);
-  st->gemm_ws = reinterpret_cast<float*>(w + w_gws);
-  st->gemm_ws_bytes = gws;
-  st->gemm_cnt = reinterpret_cast<int*>(w + w_gcnt);
-  st->gemm_cnt_n = gcnt;
+  st->part = reinterpret_cast<float*>(w + w_part);
+  st->part_bytes = pbytes;
   st->part_val = reinterpret_cast<float*>(w + w_pv);
   st->part_idx = reinterpret_cast<int*>(w + w_pi);
   if (cudaMemset(st->ws, 0, off) != cudaSuccess || cudaMemset(st->base, 0, o_done + l.done) != cudaSuccess) {
@@ -310,13 +300,17 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
   int rc;
   auto plan = [&](GemmOp* op, const void* X, int Mx, int K, const void* const* W, const int* rows,
                   int nseg, int mode, void* Y, int ldy) {
-    return gemm_plan(op, dt, X, Mx, K, W, rows, nseg, mode, Y, ldy, st->gemm_ws, st->gemm_ws_bytes,
-                     st->gemm_cnt, st->gemm_cnt_n, st->err, st->num_sms, 0);
+    const int r = gemm_plan(op, dt, X, Mx, K, W, rows, nseg, mode, Y, ldy, st->err, st->num_sms, 0, 0);
+    if (r == LSP_OK && mode == EPI_PARTIAL &&
+        (size_t)op->p.splits * Mx * op->p.N * sizeof(float) > st->part_bytes)
+      return LSP_ERR_SHAPE;
+    return r;
   };
   {
     const void* W[1] = {w->fuse};
     const int rows[1] = {c.H};
-    if ((rc = plan(&st->fuse, st->h, c.C, c.L * c.H, W, rows, 1, EPI_F32, st->c, c.H)) != LSP_OK) return rc;
+    if ((rc = plan(&st->fuse, st->h, c.C, c.L * c.H, W, rows, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
+      return rc;
   }
   for (int j = 0; j < c.D; ++j) {
     const lsp_layer_weights& lw = w->layer[j];
@@ -325,12 +319,12 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
       return LSP_ERR_ARG;
     const void* Wqkv[3] = {lw.wq, lw.wk, lw.wv};
     const int rqkv[3] = {c.nq * c.d, c.nkv * c.d, c.nkv * c.d};
-    if ((rc = plan(&st->qkv_op[j], st->xn, M, c.H, Wqkv, rqkv, 3, EPI_T, st->qkv,
+    if ((rc = plan(&st->qkv_op[j], st->xn, M, c.H, Wqkv, rqkv, 3, EPI_PARTIAL, st->part,
                    (c.nq + 2 * c.nkv) * c.d)) != LSP_OK)
       return rc;
     const void* Wo[1] = {lw.wo};
     const int ro[1] = {c.H};
-    if ((rc = plan(&st->o_op[j], st->o, M, c.nq * c.d, Wo, ro, 1, EPI_RESID, st->x, c.H)) != LSP_OK)
+    if ((rc = plan(&st->o_op[j], st->o, M, c.nq * c.d, Wo, ro, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
       return rc;
     const void* Wgu[2] = {lw.w_gate, lw.w_up};
     const int rgu[2] = {c.F, c.F};
@@ -338,7 +332,7 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
       return rc;
     const void* Wd[1] = {lw.w_down};
     const int rd[1] = {c.H};
-    if ((rc = plan(&st->down_op[j], st->act, M, c.F, Wd, rd, 1, EPI_RESID, st->x, c.H)) != LSP_OK)
+    if ((rc = plan(&st->down_op[j], st->act, M, c.F, Wd, rd, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
       return rc;
   }
   {
@@ -390,7 +384,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   // input slots + first input norm + rotary table
   CombineParams cp;
   cp.tokens = block_tokens; cp.embed = w->embed; cp.pos = w->pos; cp.mask_emb = w->mask_emb;
-  cp.c = st->c; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
+  cp.c = st->part; cp.c_splits = st->fuse.p.splits; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
   cp.t = st->t; cp.err = st->err; cp.C = c.C; cp.B = c.B; cp.H = c.H; cp.V = c.V; cp.d = c.d;
   cp.eps = c.rms_eps; cp.theta = (double)c.rope_theta;
   if ((rc = launch_combine(cp, c.dtype, s)) != LSP_OK) return rc;
@@ -400,7 +394,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     if ((rc = gemm_launch(&st->qkv_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
     AttnParams ap;
-    ap.qkv = st->qkv; ap.q_norm = lw.q_norm; ap.k_norm = lw.k_norm; ap.rope = st->rope;
+    ap.qkv = st->part; ap.qkv_splits = st->qkv_op[j].p.splits; ap.q_norm = lw.q_norm; ap.k_norm = lw.k_norm; ap.rope = st->rope;
     ap.win_k = st->win_k; ap.win_v = st->win_v; ap.G = st->G; ap.m = st->m; ap.t = st->t;
     ap.out = st->o; ap.C = c.C; ap.B = c.B; ap.L = c.L; ap.nq = c.nq; ap.nkv = c.nkv; ap.d = c.d;
     ap.W = c.W; ap.R = c.R; ap.layer = c.layer_map[j]; ap.eps = c.rms_eps;
@@ -408,7 +402,8 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->o_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
-    if ((rc = launch_rmsnorm(st->x, lw.post_norm, st->xn, M, c.H, c.rms_eps, c.dtype, s)) != LSP_OK)
+    if ((rc = launch_resid_norm(st->x, st->part, st->o_op[j].p.splits, lw.post_norm, st->xn, M, c.H,
+                                c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->gu_op[j], s)) != LSP_OK) return rc;
@@ -416,7 +411,8 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     if ((rc = gemm_launch(&st->down_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
     const void* next_norm = j + 1 < c.D ? w->layer[j + 1].in_norm : w->final_norm;
-    if ((rc = launch_rmsnorm(st->x, next_norm, st->xn, M, c.H, c.rms_eps, c.dtype, s)) != LSP_OK)
+    if ((rc = launch_resid_norm(st->x, st->part, st->down_op[j].p.splits, next_norm, st->xn, M, c.H,
+                                c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
   }
@@ -439,9 +435,7 @@ int lsp_sample(lsp_state* st, const float* base_logits, const int32_t* prev_toke
 
 size_t lsp_linear_workspace_bytes(int M, int N, int splits) {
   if (M < 1 || N < 1 || splits < 1) return 0;
-  const int rows[1] = {N};
-  const int tiles = gemm_tiles(EPI_F32, rows, 1);
-  return align256((size_t)tiles * 4) + gemm_ws_bytes(M, tiles, splits);
+  return splits == 1 ? 0 : (size_t)splits * M * N * sizeof(float);
 }
 
 int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype, int splits,
@@ -449,26 +443,21 @@ int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int 
   if (!X || !W || !Y || M < 1 || N < 1 || K < 1 || splits < 1 || splits > 16) return LSP_ERR_ARG;
   if (dtype != LSP_DTYPE_BF16 && dtype != LSP_DTYPE_F32) return LSP_ERR_ARG;
   const int rows[1] = {N};
-  const int tiles = gemm_tiles(EPI_F32, rows, 1);
-  int* cnt = nullptr;
-  float* ws = nullptr;
-  size_t ws_bytes = 0;
-  if (splits > 1) {
-    if (!workspace || workspace_bytes < lsp_linear_workspace_bytes(M, N, splits)) return LSP_ERR_ARG;
-    cnt = static_cast<int*>(workspace);
-    ws = reinterpret_cast<float*>(static_cast<char*>(workspace) + align256((size_t)tiles * 4));
-    ws_bytes = workspace_bytes - align256((size_t)tiles * 4);
-  }
+  if (splits > 1 && (!workspace || workspace_bytes < lsp_linear_workspace_bytes(M, N, splits)))
+    return LSP_ERR_ARG;
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return LSP_ERR_CUDA;
   GemmOp op;
   const void* Ws[1] = {W};
-  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, EPI_F32, Y, N, ws, ws_bytes, cnt, tiles,
-                     nullptr, sms, splits);
+  float* part = static_cast<float*>(workspace);
+  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, splits > 1 ? EPI_PARTIAL : EPI_F32,
+                     splits > 1 ? part : Y, N, nullptr, sms, splits, 0);
   if (rc != LSP_OK) return rc;
-  return gemm_launch(&op, S(stream));
+  if (op.p.splits != splits) return LSP_ERR_SHAPE;
+  if ((rc = gemm_launch(&op, S(stream))) != LSP_OK || splits == 1) return rc;
+  return launch_sum_partials(part, splits, (size_t)M * N, Y, S(stream));
 }
 
 int lsp_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint32_t* out,

@@ -10,12 +10,32 @@
 
 namespace lsp {
 
+// ------------------------------------------------------------------ launch helper
+// Launch as a programmatic dependent of the preceding work in the stream: the
+// kernel may start while its predecessor finishes and must call griddep_wait()
+// before it reads the predecessor's outputs or writes anything it reads.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ------------------------------------------------------------------ GEMM
 enum EpiMode {
-  EPI_F32 = 0,     // Y (float) = acc
-  EPI_T = 1,       // Y (dtype) = acc
-  EPI_RESID = 2,   // Y (float) += acc
-  EPI_SWIGLU = 3,  // Y (dtype) = silu(acc_gate) * acc_up
+  EPI_F32 = 0,      // Y (float) = acc
+  EPI_T = 1,        // Y (dtype) = acc
+  EPI_PARTIAL = 2,  // Y (float) [split][M][ldy] = this split's partial sum (the consumer adds)
+  EPI_SWIGLU = 3,   // Y (dtype) = silu(acc_gate) * acc_up
 };
 
 constexpr int kGemmThreads = 192;   // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
@@ -24,14 +44,13 @@ constexpr int kTileRows = 128;      // weight rows per tile (UMMA M)
 struct GemmParams {
   int M, N, K;          // token rows, output features, reduction length
   int kblocks, splits, n_tiles;
+  int wt;               // weight tiles per CTA (they share the activation tile)
   int mode;
   int seg_tile0[3];     // first tile index of each A segment
   int nseg;
-  int bn, n_tok_tiles, m_pad, stages, tmem_cols;
+  int bn, n_tok_tiles, m_pad, stages, tmem_cols, pd;
   void* Y;
   int ldy;
-  float* ws;
-  int* counters;
   unsigned* err;
 };
 
@@ -46,15 +65,20 @@ struct GemmOp {
 
 // Plan Y = X W^T where W is the row-concatenation of `nseg` weight segments
 // (each [seg_rows[i]][K]); for EPI_SWIGLU, segment 0 = gate and 1 = up, both
-// [N][K].  splits <= 0 picks a split-K factor for `num_sms`.
+// [N][K].  EPI_PARTIAL writes `splits` partial sums [splits][M][ldy]; other
+// modes need splits == 1.  splits <= 0 / wt <= 0 choose for `num_sms`.
 int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
-              const int* seg_rows, int nseg, int mode, void* Y, int ldy, float* ws,
-              size_t ws_bytes, int* counters, int n_counters, unsigned* err, int num_sms,
-              int splits);
+              const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
+              int num_sms, int splits, int wt);
 int gemm_launch(const GemmOp* op, cudaStream_t s);
-size_t gemm_ws_bytes(int M, int n_tiles, int splits);
+// The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 = choose).
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
-int gemm_auto_splits(int n_tiles, int kblocks, int num_sms);
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost);
+double gemm_partial_cost(int M);
+int gemm_kblocks(int K, int dtype);
+// Deterministic sum of `splits` fp32 partials [splits][n] into y[n].
+int launch_sum_partials(const float* part, int splits, size_t n, float* y, cudaStream_t s);
 
 // ------------------------------------------------------------------ view update
 struct ViewParams {
@@ -82,7 +106,8 @@ struct CombineParams {
   const void* embed;       // [V][H]
   const void* pos;         // [B][H]
   const void* mask_emb;    // [H]
-  const float* c;          // [C][H]
+  const float* c;          // [splits][C][H] partial sums of c_t
+  int c_splits;
   const void* norm_w;      // [H] first layer input norm
   float* x;                // [M][H]
   void* xn;                // [M][H]
@@ -94,12 +119,14 @@ struct CombineParams {
   double theta;
 };
 int launch_combine(const CombineParams& p, int dtype, cudaStream_t s);
-int launch_rmsnorm(const float* x, const void* w, void* out, int M, int H, float eps, int dtype,
-                   cudaStream_t s);
+// x += sum_s part[s] (s < splits, fp32 [splits][M][H]); out = RMSNorm(x) * w.
+int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
+                      int H, float eps, int dtype, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention
 struct AttnParams {
-  const void* qkv;        // [M][(nq+2nkv)d] projections (pre-norm, pre-rotary)
+  const float* qkv;       // [splits][M][(nq+2nkv)d] fp32 partial sums of the projections
+  int qkv_splits;
   const void* q_norm;     // [d]
   const void* k_norm;     // [d]
   const float* rope;      // [C][B][d/2][2]
