@@ -163,28 +163,39 @@ __global__ void __launch_bounds__(512)
         src = qkv + mrow + (size_t)(p.nq + p.nkv + g) * kHD;
         dst = sVbw + (size_t)i * row;
       }
-      float x[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        float acc = src[lane + 32 * e];
-        for (int sp = 1; sp < p.qkv_splits; ++sp) acc += src[sp * pstride + lane + 32 * e];
-        x[e] = acc;
+      // lane holds elements 4*lane .. 4*lane+3; the rotary partner of element f
+      // (f < 64) is f + 64, held by lane ^ 16
+      float4 x = reinterpret_cast<const float4*>(src)[lane];
+      for (int sp = 1; sp < p.qkv_splits; ++sp) {
+        const float4 y = reinterpret_cast<const float4*>(src + sp * pstride)[lane];
+        x.x += y.x; x.y += y.y; x.z += y.z; x.w += y.w;
       }
       if (kind <= rep) {
         const bf16* w = kind < rep ? qn : kn;
-        const float ss = warp_sum(x[0] * x[0] + x[1] * x[1] + x[2] * x[2] + x[3] * x[3]);
+        const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
         const float rstd = rsqrtf(ss / (float)kHD + p.eps);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) x[e] *= rstd * to_f(w[lane + 32 * e]);
-        const float* cs = p.rope + (size_t)(b * B + i) * (kHD / 2) * 2;
-        const float c0 = cs[2 * lane], s0 = cs[2 * lane + 1];
-        const float c1 = cs[2 * (lane + 32)], s1 = cs[2 * (lane + 32) + 1];
-        const float y0 = x[0] * c0 - x[2] * s0, y2 = x[2] * c0 + x[0] * s0;
-        const float y1 = x[1] * c1 - x[3] * s1, y3 = x[3] * c1 + x[1] * s1;
-        x[0] = y0; x[1] = y1; x[2] = y2; x[3] = y3;
+        const uint2 wr = reinterpret_cast<const uint2*>(w)[lane];
+        const float2 w01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wr.x));
+        const float2 w23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wr.y));
+        x.x *= rstd * w01.x; x.y *= rstd * w01.y; x.z *= rstd * w23.x; x.w *= rstd * w23.y;
+        float4 q;
+        q.x = __shfl_xor_sync(0xffffffffu, x.x, 16);
+        q.y = __shfl_xor_sync(0xffffffffu, x.y, 16);
+        q.z = __shfl_xor_sync(0xffffffffu, x.z, 16);
+        q.w = __shfl_xor_sync(0xffffffffu, x.w, 16);
+        const float4* cs = reinterpret_cast<const float4*>(p.rope + ((size_t)(b * B + i) * (kHD / 2) + (lane & 15) * 4) * 2);
+        const float4 c01 = cs[0], c23 = cs[1];      // (cos, sin) of f, f+1 / f+2, f+3
+        const float sg = lane < 16 ? -1.f : 1.f;
+        x.x = x.x * c01.x + sg * q.x * c01.y;
+        x.y = x.y * c01.z + sg * q.y * c01.w;
+        x.z = x.z * c23.x + sg * q.z * c23.y;
+        x.w = x.w * c23.z + sg * q.w * c23.w;
       }
-#pragma unroll
-      for (int e = 0; e < 4; ++e) dst[lane + 32 * e] = __float2bfloat16_rn(x[e]);
+      const __nv_bfloat162 o01 = __floats2bfloat162_rn(x.x, x.y), o23 = __floats2bfloat162_rn(x.z, x.w);
+      uint2 ov;
+      ov.x = *reinterpret_cast<const uint32_t*>(&o01);
+      ov.y = *reinterpret_cast<const uint32_t*>(&o23);
+      *reinterpret_cast<uint2*>(dst + 4 * lane) = ov;
     }
   }
   cp_async_wait_all();

@@ -38,9 +38,11 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   return c;
 }
 
+// g = -log(-log u): the inner log keeps full relative accuracy (u can be within
+// 2^-24 of 1, where -log u is tiny); the outer log only needs absolute accuracy.
 __device__ __forceinline__ float gumbel_of(uint32_t x) {
   const float u = ((float)(x >> 9) + 0.5f) * 1.1920928955078125e-07f;   // 2^-23
-  return -logf(-logf(u));
+  return -__logf(-logf(u));
 }
 
 __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
@@ -55,15 +57,16 @@ __device__ __forceinline__ void mma_bf16_s(float* c, const uint32_t* a, uint32_t
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// argmax over the previous step's per-CTA partials of request b (one warp)
+// argmax over the previous step's per-CTA partials of request b (one warp);
+// partials are laid out [buf][b][block] so the lanes read consecutive blocks.
 __device__ __forceinline__ int resolve_prev(const SampleParams& p, int buf, int b, int lane) {
   float bv = -INFINITY;
   int bi = 0x7fffffff;
-  const float* pv = p.part_val + (size_t)buf * p.nblk * p.C;
-  const int* pi = p.part_idx + (size_t)buf * p.nblk * p.C;
+  const float* pv = p.part_val + ((size_t)buf * p.C + b) * p.nblk;
+  const int* pi = p.part_idx + ((size_t)buf * p.C + b) * p.nblk;
   for (int gblk = lane; gblk < p.nblk; gblk += 32) {
-    const float v = pv[(size_t)gblk * p.C + b];
-    const int i = pi[(size_t)gblk * p.C + b];
+    const float v = pv[gblk];
+    const int i = pi[gblk];
     if (better(v, i, bv, bi)) { bv = v; bi = i; }
   }
 #pragma unroll
@@ -75,8 +78,9 @@ __device__ __forceinline__ int resolve_prev(const SampleParams& p, int buf, int 
   return bi;
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kSampThreads) sample_step_kernel(const SampleParams p, const int step) {
+// KG = ceil(4 * C / 32): groups of four vocabulary entries each lane handles per tile.
+template <typename T, int KG>
+__global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const SampleParams p, const int step) {
   extern __shared__ __align__(16) uint8_t ssm_raw[];
   const int C = p.C, rc = p.rc;
   const int C8 = (C + 7) / 8 * 8;
@@ -121,81 +125,102 @@ __global__ void __launch_bounds__(kSampThreads) sample_step_kernel(const SampleP
 
   const T* Wc = static_cast<const T*>(p.Wc);
   const uint2 key = make_uint2((uint32_t)p.seed, (uint32_t)(p.seed >> 32));
-  const float inv_t = p.temperature > 0.f ? p.temperature : 1.f;
-  const bool sample = p.temperature > 0.f;
+  const float temp = p.temperature;
+  const bool sample = temp > 0.f;
   float* cw = corr_s + (size_t)warp * kMaxC * 17;
-  float bv[kMaxC / 8];
-  int bi[kMaxC / 8];
+  float bv[KG];
+  int bi[KG];
 #pragma unroll
-  for (int k = 0; k < kMaxC / 8; ++k) { bv[k] = -INFINITY; bi[k] = 0x7fffffff; }
+  for (int k = 0; k < KG; ++k) { bv[k] = -INFINITY; bi[k] = 0x7fffffff; }
 
   const int ntiles = p.V / 16;
-  for (int tile = blockIdx.x * kSampWarps + warp; tile < ntiles; tile += gridDim.x * kSampWarps) {
+  const int stride = gridDim.x * kSampWarps;
+  auto zoff = [&](int tile, int k) {
+    const int gi = lane + 32 * k;
+    return ((size_t)(gi >> 2) * p.B + step) * p.V + tile * 16 + 4 * (gi & 3);
+  };
+  float4 zc[KG], zn[KG];
+  int tile = blockIdx.x * kSampWarps + warp;
+#pragma unroll
+  for (int k = 0; k < KG; ++k)
+    if (tile < ntiles && lane + 32 * k < 4 * C) zc[k] = *reinterpret_cast<const float4*>(p.src + zoff(tile, k));
+  for (; tile < ntiles; tile += stride) {
+    const int next = tile + stride;
+#pragma unroll
+    for (int k = 0; k < KG; ++k)
+      if (next < ntiles && lane + 32 * k < 4 * C) zn[k] = *reinterpret_cast<const float4*>(p.src + zoff(next, k));
     const int v0 = tile * 16;
     // correction W_c[v0:v0+16] . E_c(y)^T for all requests -> cw[b][v]
     if constexpr (sizeof(T) == 2) {
       const bf16* es = reinterpret_cast<const bf16*>(e_s);
       const bf16* wr = reinterpret_cast<const bf16*>(Wc) + (size_t)(v0 + (lane >> 2)) * rc + (lane & 3) * 2;
-      for (int nt = 0; nt < C8 / 8; ++nt) {
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        const bf16* er = es + (size_t)(nt * 8 + (lane >> 2)) * lde + (lane & 3) * 2;
-        for (int kk = 0; kk < rc / 16; ++kk) {
-          uint32_t a[4];
-          a[0] = *reinterpret_cast<const uint32_t*>(wr + kk * 16);
-          a[1] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16);
-          a[2] = *reinterpret_cast<const uint32_t*>(wr + kk * 16 + 8);
-          a[3] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16 + 8);
-          const uint32_t b0 = *reinterpret_cast<const uint32_t*>(er + kk * 16);
-          const uint32_t b1 = *reinterpret_cast<const uint32_t*>(er + kk * 16 + 8);
-          mma_bf16_s(acc, a, b0, b1);
+      float acc[KG][4];                                     // KG = ceil(C / 8) n-tiles of 8 requests
+#pragma unroll
+      for (int nt = 0; nt < KG; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+      for (int kk = 0; kk < rc / 16; ++kk) {
+        uint32_t a[4];
+        a[0] = *reinterpret_cast<const uint32_t*>(wr + kk * 16);
+        a[1] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16);
+        a[2] = *reinterpret_cast<const uint32_t*>(wr + kk * 16 + 8);
+        a[3] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16 + 8);
+#pragma unroll
+        for (int nt = 0; nt < KG; ++nt) {
+          const bf16* er = es + (size_t)(nt * 8 + (lane >> 2)) * lde + (lane & 3) * 2 + kk * 16;
+          mma_bf16_s(acc[nt], a, *reinterpret_cast<const uint32_t*>(er),
+                     *reinterpret_cast<const uint32_t*>(er + 8));
         }
+      }
+#pragma unroll
+      for (int nt = 0; nt < KG; ++nt) {
         const int bcol = nt * 8 + (lane & 3) * 2, vr = lane >> 2;
-        if (bcol < C) { cw[bcol * 17 + vr] = acc[0]; cw[bcol * 17 + vr + 8] = acc[2]; }
-        if (bcol + 1 < C) { cw[(bcol + 1) * 17 + vr] = acc[1]; cw[(bcol + 1) * 17 + vr + 8] = acc[3]; }
+        if (bcol < C) { cw[bcol * 17 + vr] = acc[nt][0]; cw[bcol * 17 + vr + 8] = acc[nt][2]; }
+        if (bcol + 1 < C) { cw[(bcol + 1) * 17 + vr] = acc[nt][1]; cw[(bcol + 1) * 17 + vr + 8] = acc[nt][3]; }
       }
     } else {
       for (int idx = lane; idx < 16 * C; idx += 32) {
         const int v = idx & 15, b = idx >> 4;
-        const T* wr = Wc + (size_t)(v0 + v) * rc;
+        const T* wrow = Wc + (size_t)(v0 + v) * rc;
         const T* er = e_s + (size_t)b * lde;
         float acc = 0.f;
-        for (int r = 0; r < rc; ++r) acc = fmaf(to_f(wr[r]), to_f(er[r]), acc);
+        for (int r = 0; r < rc; ++r) acc = fmaf(to_f(wrow[r]), to_f(er[r]), acc);
         cw[b * 17 + v] = acc;
       }
     }
     __syncwarp();
     // corrected logits, noise and running argmax: lane handles groups of 4 entries
 #pragma unroll
-    for (int k = 0; k < kMaxC / 8; ++k) {
+    for (int k = 0; k < KG; ++k) {
       const int gi = lane + 32 * k;
-      if (gi >= 4 * C) break;
-      const int b = gi >> 2, vq = gi & 3;
-      const int v = v0 + 4 * vq;
-      const size_t off = ((size_t)b * p.B + step) * p.V + v;
-      float4 z = *reinterpret_cast<const float4*>(p.src + off);
-      z.x += cw[b * 17 + 4 * vq + 0];
-      z.y += cw[b * 17 + 4 * vq + 1];
-      z.z += cw[b * 17 + 4 * vq + 2];
-      z.w += cw[b * 17 + 4 * vq + 3];
-      if (p.dst) *reinterpret_cast<float4*>(p.dst + off) = z;
-      float sc[4] = {z.x, z.y, z.z, z.w};
-      if (sample) {
-        const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)step, (uint32_t)b, p.round), key);
-        sc[0] = sc[0] / inv_t + gumbel_of(x.x);
-        sc[1] = sc[1] / inv_t + gumbel_of(x.y);
-        sc[2] = sc[2] / inv_t + gumbel_of(x.z);
-        sc[3] = sc[3] / inv_t + gumbel_of(x.w);
-      }
+      if (gi < 4 * C) {
+        const int b = gi >> 2, vq = gi & 3;
+        const int v = v0 + 4 * vq;
+        float4 z = zc[k];
+        z.x += cw[b * 17 + 4 * vq + 0];
+        z.y += cw[b * 17 + 4 * vq + 1];
+        z.z += cw[b * 17 + 4 * vq + 2];
+        z.w += cw[b * 17 + 4 * vq + 3];
+        if (p.dst) *reinterpret_cast<float4*>(p.dst + zoff(tile, k)) = z;
+        float sc[4] = {z.x, z.y, z.z, z.w};
+        if (sample) {
+          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)step, (uint32_t)b, p.round), key);
+          sc[0] = sc[0] / temp + gumbel_of(x.x);
+          sc[1] = sc[1] / temp + gumbel_of(x.y);
+          sc[2] = sc[2] / temp + gumbel_of(x.z);
+          sc[3] = sc[3] / temp + gumbel_of(x.w);
+        }
 #pragma unroll
-      for (int e = 0; e < 4; ++e)
-        if (better(sc[e], v + e, bv[k], bi[k])) { bv[k] = sc[e]; bi[k] = v + e; }
+        for (int e = 0; e < 4; ++e)
+          if (better(sc[e], v + e, bv[k], bi[k])) { bv[k] = sc[e]; bi[k] = v + e; }
+      }
     }
     __syncwarp();
+#pragma unroll
+    for (int k = 0; k < KG; ++k) zc[k] = zn[k];
   }
 
   // ---- per-CTA partial argmax of every request
 #pragma unroll
-  for (int k = 0; k < kMaxC / 8; ++k) {
+  for (int k = 0; k < KG; ++k) {
 #pragma unroll
     for (int o = 1; o <= 2; o <<= 1) {
       const float ov = __shfl_xor_sync(0xffffffffu, bv[k], o);
@@ -217,7 +242,7 @@ __global__ void __launch_bounds__(kSampThreads) sample_step_kernel(const SampleP
         v = red_v[w * kMaxC + b];
         i = red_i[w * kMaxC + b];
       }
-    const size_t o = ((size_t)(step & 1) * p.nblk + blockIdx.x) * C + b;
+    const size_t o = ((size_t)(step & 1) * C + b) * p.nblk + blockIdx.x;
     p.part_val[o] = v;
     p.part_idx[o] = i;
   }
@@ -250,21 +275,35 @@ static size_t sample_smem(int rc, int es) {
          (size_t)kSampWarps * kMaxC * 17 * sizeof(float) + (size_t)kMaxC * (rc + 8) * es;
 }
 
+template <typename T, int KG>
+static cudaError_t launch_step(const SampleParams& p, int step, size_t smem, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(sample_step_kernel<T, KG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)sample_smem(256, 4));
+    attr = true;
+  }
+  return launch_pdl(sample_step_kernel<T, KG>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step);
+}
+
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
   const size_t smem = sample_smem(p.rc, es);
-  static bool attr_set = false;
-  if (!attr_set) {
-    const int mx = (int)std::max(sample_smem(256, 4), sample_smem(256, 2));
-    cudaFuncSetAttribute(sample_step_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-    cudaFuncSetAttribute(sample_step_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-    attr_set = true;
-  }
+
+  const int kg = (4 * p.C + 31) / 32;
   for (int step = 0; step < p.B; ++step) {
-    cudaError_t e = dtype == LSP_DTYPE_BF16
-                        ? launch_pdl(sample_step_kernel<bf16>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step)
-                        : launch_pdl(sample_step_kernel<float>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step);
+    cudaError_t e;
+    if (dtype == LSP_DTYPE_BF16)
+      e = kg <= 1 ? launch_step<bf16, 1>(p, step, smem, s)
+        : kg <= 2 ? launch_step<bf16, 2>(p, step, smem, s)
+        : kg <= 4 ? launch_step<bf16, 4>(p, step, smem, s)
+                  : launch_step<bf16, 8>(p, step, smem, s);
+    else
+      e = kg <= 1 ? launch_step<float, 1>(p, step, smem, s)
+        : kg <= 2 ? launch_step<float, 2>(p, step, smem, s)
+        : kg <= 4 ? launch_step<float, 4>(p, step, smem, s)
+                  : launch_step<float, 8>(p, step, smem, s);
     if (e != cudaSuccess) return LSP_ERR_CUDA;
   }
   if (launch_pdl(sample_final_kernel, dim3(1), dim3(kSampThreads), 0, s, p) != cudaSuccess)

@@ -37,6 +37,29 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return s;
 }
 
+// four consecutive elements as fp32 (16-byte fp32 or 8-byte bf16 accesses)
+__device__ __forceinline__ float4 ld4(const float* p, int i4) { return reinterpret_cast<const float4*>(p)[i4]; }
+__device__ __forceinline__ float4 ld4(const bf16* p, int i4) {
+  const uint2 r = reinterpret_cast<const uint2*>(p)[i4];
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+__device__ __forceinline__ void st4(float* p, int i4, float4 v) { reinterpret_cast<float4*>(p)[i4] = v; }
+__device__ __forceinline__ void st4(bf16* p, int i4, float4 v) {
+  const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 r;
+  r.x = *reinterpret_cast<const uint32_t*>(&a);
+  r.y = *reinterpret_cast<const uint32_t*>(&b);
+  reinterpret_cast<uint2*>(p)[i4] = r;
+}
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float dot4(float4 a) { return a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w; }
+
+constexpr int kMaxVec = kMaxPerThread / 4;   // float4 per thread (H <= 8192)
+
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParams p) {
   __shared__ float red[32];
@@ -78,27 +101,31 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   const T* pos = static_cast<const T*>(p.pos) + (size_t)i * p.H;
   const size_t cstride = (size_t)p.C * p.H;
   const float* c = p.c + (size_t)b * p.H;
-  float xv[kMaxPerThread];
+  const int h4 = p.H / 4;
+  float4 xv[kMaxVec];
   float ss = 0.f;
 #pragma unroll
-  for (int k = 0; k < kMaxPerThread; ++k) {
-    const int h = threadIdx.x + k * kRowThreads;
-    xv[k] = 0.f;
-    if (h < p.H) {
-      float cv = c[h];
-      for (int s = 1; s < p.c_splits; ++s) cv += c[s * cstride + h];
-      xv[k] = to_f(src[h]) + to_f(pos[h]) + cv;
-      p.x[(size_t)m * p.H + h] = xv[k];
-      ss += xv[k] * xv[k];
+  for (int k = 0; k < kMaxVec; ++k) {
+    const int j = threadIdx.x + k * kRowThreads;
+    if (j < h4) {
+      float4 cv = ld4(c, j);
+      for (int s = 1; s < p.c_splits; ++s) cv = add4(cv, ld4(c + s * cstride, j));
+      xv[k] = add4(add4(ld4(src, j), ld4(pos, j)), cv);
+      st4(p.x + (size_t)m * p.H, j, xv[k]);
+      ss += dot4(xv[k]);
     }
   }
   const float rstd = rsqrtf(block_sum(ss, red) / (float)p.H + p.eps);
   const T* w = static_cast<const T*>(p.norm_w);
   T* out = static_cast<T*>(p.xn) + (size_t)m * p.H;
 #pragma unroll
-  for (int k = 0; k < kMaxPerThread; ++k) {
-    const int h = threadIdx.x + k * kRowThreads;
-    if (h < p.H) out[h] = from_f<T>(xv[k] * rstd * to_f(w[h]));
+  for (int k = 0; k < kMaxVec; ++k) {
+    const int j = threadIdx.x + k * kRowThreads;
+    if (j < h4) {
+      const float4 wv = ld4(w, j);
+      st4(out, j, make_float4(xv[k].x * rstd * wv.x, xv[k].y * rstd * wv.y, xv[k].z * rstd * wv.z,
+                              xv[k].w * rstd * wv.w));
+    }
   }
 }
 
@@ -111,26 +138,40 @@ __global__ void __launch_bounds__(kRowThreads)
   griddep_wait();
   const int m = blockIdx.x;
   float* row = x + (size_t)m * H;
+  const float* prow = part + (size_t)m * H;
   const size_t pstride = (size_t)M * H;
-  float xv[kMaxPerThread];
+  const int h4 = H / 4;
+  float4 xv[kMaxVec];
   float ss = 0.f;
 #pragma unroll
-  for (int k = 0; k < kMaxPerThread; ++k) {
-    const int h = threadIdx.x + k * kRowThreads;
-    xv[k] = 0.f;
-    if (h < H) {
-      float v = row[h];
-      for (int s = 0; s < splits; ++s) v += part[s * pstride + (size_t)m * H + h];
-      xv[k] = v;
-      if (splits > 0) row[h] = v;
-      ss += v * v;
+  for (int k = 0; k < kMaxVec; ++k) {
+    const int j = threadIdx.x + k * kRowThreads;
+    if (j < h4) xv[k] = ld4(row, j);
+  }
+  for (int s = 0; s < splits; ++s) {
+#pragma unroll
+    for (int k = 0; k < kMaxVec; ++k) {
+      const int j = threadIdx.x + k * kRowThreads;
+      if (j < h4) xv[k] = add4(xv[k], ld4(prow + s * pstride, j));
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kMaxVec; ++k) {
+    const int j = threadIdx.x + k * kRowThreads;
+    if (j < h4) {
+      if (splits > 0) st4(row, j, xv[k]);
+      ss += dot4(xv[k]);
     }
   }
   const float rstd = rsqrtf(block_sum(ss, red) / (float)H + eps);
 #pragma unroll
-  for (int k = 0; k < kMaxPerThread; ++k) {
-    const int h = threadIdx.x + k * kRowThreads;
-    if (h < H) out[(size_t)m * H + h] = from_f<T>(xv[k] * rstd * to_f(w[h]));
+  for (int k = 0; k < kMaxVec; ++k) {
+    const int j = threadIdx.x + k * kRowThreads;
+    if (j < h4) {
+      const float4 wv = ld4(w, j);
+      st4(out + (size_t)m * H, j, make_float4(xv[k].x * rstd * wv.x, xv[k].y * rstd * wv.y,
+                                              xv[k].z * rstd * wv.z, xv[k].w * rstd * wv.w));
+    }
   }
 }
 
