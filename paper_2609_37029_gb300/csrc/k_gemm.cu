@@ -349,27 +349,41 @@ static int tuning(const char* name) {
   return v ? std::atoi(v) : 0;
 }
 
-double gemm_partial_cost(int M) {
-  int bn, ntt;
-  token_tiling(M, &bn, &ntt);
-  return (double)(bn * ntt) / 64.0;
+// Two 2-stage CTAs per SM keep the tensor pipe fed from two MMA issuers and
+// overlap one CTA's prologue/epilogue with the other's weight stream; the pair
+// must fit one SM's shared memory and TMEM.
+static bool two_per_sm_fits(int wt, int m_pad) {
+  const int stage_bytes = wt * (int)kTileBytes + m_pad * 128;
+  return 2 * stage_bytes + 2048 <= kSmemBudget / 2 && 2 * wt * m_pad <= 512;
 }
 
-// split-K factor: minimise waves x (k-blocks per CTA + fixed per-CTA overhead)
-// (partial_cost: the per-CTA cost of writing and re-reading one fp32 partial,
-// in k-block units)
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost) {
+static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
+  return ctas * 4 >= (long long)num_sms * 5 && two_per_sm_fits(wt, m_pad);
+}
+
+// Split-K factor from a cost model in units of one k-block of one of two
+// co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
+// fixed per-CTA cost) + the consumer's re-read of the fp32 split partials
+// from L2 (partial_cost per split).  A lone CTA on an SM streams a k-block in
+// ~0.63 of that time.
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok) {
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(16, kblocks); ++s) {
     const long long ctas = (long long)n_ctas * s;
-    const long long waves = (ctas + num_sms - 1) / num_sms;
-    const double per = (double)((kblocks + s - 1) / s) + 4.0 + (s > 1 ? partial_cost : 0.0);
-    const double cost = (double)waves * per;
+    const bool two = two_ok && ctas * 4 >= (long long)num_sms * 5;
+    const long long slots = two ? 2LL * num_sms : num_sms;
+    const long long waves = (ctas + slots - 1) / slots;
+    const double per = (double)((kblocks + s - 1) / s) * (two ? 1.0 : 0.63) + 2.0;
+    const double cost = (double)waves * per + (s > 1 ? partial_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
   return splits;
 }
+
+// Consumer cost of one M x N fp32 partial read back from L2 (~5 TB/s), in the
+// model's k-block units (~1.56 us).
+double gemm_partial_cost(int M, int N) { return (double)M * N * 4.0 / 5e12 / 1.56e-6; }
 
 void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt) {
   int bn, ntt;
@@ -380,7 +394,10 @@ void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, in
   const int kblocks = gemm_kblocks(K, dtype);
   const int n_ctas = (n_tiles + *wt - 1) / *wt;
   if (*splits <= 0)
-    *splits = mode == EPI_PARTIAL ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M)) : 1;
+    *splits = mode == EPI_PARTIAL
+                  ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows),
+                                     two_per_sm_fits(*wt, m_pad))
+                  : 1;
   *splits = std::max(1, std::min(*splits, kblocks));
 }
 
@@ -424,14 +441,12 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   const int stage_bytes = wt * (int)kTileBytes + p.m_pad * 128;
   p.stages = std::min(8, (kSmemBudget - 2048) / stage_bytes);
   const int n_ctas = (p.n_tiles + wt - 1) / wt;
-  // With CTAs to spare, two 2-stage CTAs per SM beat one deep CTA: one CTA's
-  // prologue and epilogue overlap the other's weight stream (same bytes in flight).
-  if ((long long)n_ctas * splits >= (long long)num_sms * 5 / 4 && 2 * stage_bytes + 2048 <= kSmemBudget / 2 &&
-      2 * wt * p.m_pad <= 512)
-    p.stages = 2;
+  if (use_two_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad)) p.stages = 2;
   if (tuning("LSP_GEMM_STAGES") > 0) p.stages = std::min(p.stages, tuning("LSP_GEMM_STAGES"));
   if (p.stages < 2) return LSP_ERR_SHAPE;
-  p.pd = 0;                             // weight k-blocks prefetched into L2 ahead (off: it re-read DRAM)
+  // L2 prefetch of each weight tile issued before waiting for its smem slot
+  // (distance 1: 318 -> 281 us at the LM-head shape; longer distances were slower)
+  p.pd = 1;
   if (std::getenv("LSP_GEMM_PD")) p.pd = std::max(0, tuning("LSP_GEMM_PD"));
   if (splits > 1 && mode != EPI_PARTIAL) return LSP_ERR_SHAPE;
   p.splits = splits;
