@@ -136,7 +136,8 @@ typedef struct lsp_weights {
 /*
  * Sampling of the proposals (Eq. proposal-factorization).  temperature == 0:
  * greedy, y_i = argmax_v z_i[v].  temperature > 0: Gumbel-max,
- * y_i = argmax_v (z_i[v] / T + g), g = -log(-log u), u = ((x >> 9) + 0.5) * 2^-23,
+ * y_i = argmax_v (z_i[v] / T + g) (z / T taken in fp32 as z * fl(1/T), exact at T = 1),
+ * g = -log(-log u), u = ((x >> 9) + 0.5) * 2^-23,
  * x = word (v & 3) of Philox4x32-10 with key (seed lo32, seed hi32) and counter
  * (v >> 2, i, b, round).  Ties go to the lowest vocabulary index.
  */

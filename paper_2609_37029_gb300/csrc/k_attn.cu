@@ -139,19 +139,16 @@ __global__ void __launch_bounds__(512)
     const int hh = hr / (16 - B), i = B + hr % (16 - B);
     *reinterpret_cast<uint4*>(sQ + (size_t)(hh * 16 + i) * row + c) = make_uint4(0, 0, 0, 0);
   }
-  // ---- block q (rep heads), k, v of KV head g (sum of the projection's split-K
-  //      partials): per-head RMSNorm + rotary for q, k
+  // ---- block q (rep heads), k, v of KV head g, already normalised and rotated
   {
-    const float* qkv = p.qkv;
+    const bf16* qkv = static_cast<const bf16*>(p.qkv);
     const int ldq = (p.nq + 2 * p.nkv) * kHD;
-    const size_t pstride = (size_t)p.C * B * ldq;
-    const bf16* qn = static_cast<const bf16*>(p.q_norm);
-    const bf16* kn = static_cast<const bf16*>(p.k_norm);
     const int kinds = rep + 2;
-    for (int item = warp; item < B * kinds; item += nwarps) {
+    for (int idx = tid; idx < B * kinds * 16; idx += nthr) {
+      const int c = (idx & 15) * 8, item = idx >> 4;
       const int i = item / kinds, kind = item % kinds;
       const size_t mrow = (size_t)(b * B + i) * ldq;
-      const float* src;
+      const bf16* src;
       bf16* dst;
       if (kind < rep) {
         src = qkv + mrow + (size_t)(g * rep + kind) * kHD;
@@ -163,39 +160,7 @@ __global__ void __launch_bounds__(512)
         src = qkv + mrow + (size_t)(p.nq + p.nkv + g) * kHD;
         dst = sVbw + (size_t)i * row;
       }
-      // lane holds elements 4*lane .. 4*lane+3; the rotary partner of element f
-      // (f < 64) is f + 64, held by lane ^ 16
-      float4 x = reinterpret_cast<const float4*>(src)[lane];
-      for (int sp = 1; sp < p.qkv_splits; ++sp) {
-        const float4 y = reinterpret_cast<const float4*>(src + sp * pstride)[lane];
-        x.x += y.x; x.y += y.y; x.z += y.z; x.w += y.w;
-      }
-      if (kind <= rep) {
-        const bf16* w = kind < rep ? qn : kn;
-        const float ss = warp_sum(x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w);
-        const float rstd = rsqrtf(ss / (float)kHD + p.eps);
-        const uint2 wr = reinterpret_cast<const uint2*>(w)[lane];
-        const float2 w01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wr.x));
-        const float2 w23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wr.y));
-        x.x *= rstd * w01.x; x.y *= rstd * w01.y; x.z *= rstd * w23.x; x.w *= rstd * w23.y;
-        float4 q;
-        q.x = __shfl_xor_sync(0xffffffffu, x.x, 16);
-        q.y = __shfl_xor_sync(0xffffffffu, x.y, 16);
-        q.z = __shfl_xor_sync(0xffffffffu, x.z, 16);
-        q.w = __shfl_xor_sync(0xffffffffu, x.w, 16);
-        const float4* cs = reinterpret_cast<const float4*>(p.rope + ((size_t)(b * B + i) * (kHD / 2) + (lane & 15) * 4) * 2);
-        const float4 c01 = cs[0], c23 = cs[1];      // (cos, sin) of f, f+1 / f+2, f+3
-        const float sg = lane < 16 ? -1.f : 1.f;
-        x.x = x.x * c01.x + sg * q.x * c01.y;
-        x.y = x.y * c01.z + sg * q.y * c01.w;
-        x.z = x.z * c23.x + sg * q.z * c23.y;
-        x.w = x.w * c23.z + sg * q.w * c23.w;
-      }
-      const __nv_bfloat162 o01 = __floats2bfloat162_rn(x.x, x.y), o23 = __floats2bfloat162_rn(x.z, x.w);
-      uint2 ov;
-      ov.x = *reinterpret_cast<const uint32_t*>(&o01);
-      ov.y = *reinterpret_cast<const uint32_t*>(&o23);
-      *reinterpret_cast<uint2*>(dst + 4 * lane) = ov;
+      cp_async16(dst + c, src + c);
     }
   }
   cp_async_wait_all();
@@ -335,37 +300,17 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
   float* sv = sk + B * d;
   float* ss = sv + B * d;                 // [B][ctx]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+  (void)lane;
   griddep_launch();
   griddep_wait();
-  const float* qkv = p.qkv;
+  const T* qkv = static_cast<const T*>(p.qkv);
   const int ldq = (p.nq + 2 * p.nkv) * d;
-  const size_t pstride = (size_t)p.C * B * ldq;
-  auto qkv_at = [&](const float* ptr, int e) {
-    float acc = ptr[e];
-    for (int sp = 1; sp < p.qkv_splits; ++sp) acc += ptr[sp * pstride + e];
-    return acc;
-  };
-  for (int item = warp; item < 3 * B; item += nw) {
-    const int i = item / 3, kind = item % 3;
+  for (int idx = tid; idx < 3 * B * d; idx += blockDim.x) {
+    const int kind = idx / (B * d), i = (idx / d) % B, e = idx % d;
     const size_t mrow = (size_t)(b * B + i) * ldq;
-    const float* src = qkv + mrow + (kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
-                                                                          : (size_t)(p.nq + p.nkv + g) * d);
-    float* dst = (kind == 0 ? sq : kind == 1 ? sk : sv) + i * d;
-    if (kind == 2) {
-      for (int e = lane; e < d; e += 32) dst[e] = qkv_at(src, e);
-      continue;
-    }
-    float part = 0.f;
-    for (int e = lane; e < d; e += 32) part += qkv_at(src, e) * qkv_at(src, e);
-    const float rstd = rsqrtf(warp_sum(part) / (float)d + p.eps);
-    const T* w = static_cast<const T*>(kind == 0 ? p.q_norm : p.k_norm);
-    const float* cs = p.rope + (size_t)(b * B + i) * half * 2;
-    for (int f = lane; f < half; f += 32) {
-      const float x1 = qkv_at(src, f) * rstd * to_f(w[f]);
-      const float x2 = qkv_at(src, f + half) * rstd * to_f(w[f + half]);
-      dst[f] = x1 * cs[2 * f] - x2 * cs[2 * f + 1];
-      dst[f + half] = x2 * cs[2 * f] + x1 * cs[2 * f + 1];
-    }
+    const size_t col = kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
+                                                                : (size_t)(p.nq + p.nkv + g) * d;
+    (kind == 0 ? sq : kind == 1 ? sk : sv)[i * d + e] = to_f(qkv[mrow + col + e]);
   }
   __syncthreads();
   const size_t wbase = ((size_t)(b * p.L + p.layer) * p.nkv + g) * p.W * d;
@@ -416,6 +361,77 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
     }
     out[(size_t)(b * B + i) * p.nq * d + (size_t)h * d + e] = from_f<T>(acc);
   }
+}
+
+// ------------------------------------------------------------ q/k/v finalisation
+// One warp per (block row, head): the sum of the q/k/v projection's split-K
+// partials in split order, then for q and k heads the per-head RMSNorm and the
+// rotary embedding (pairs f, f + d/2; lane l holds elements EPL*l .. EPL*l+EPL-1,
+// its rotary partner lives in lane l ^ 16).
+template <typename T, int EPL>
+__global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
+  griddep_launch();
+  griddep_wait();
+  const int heads = p.nq + 2 * p.nkv;
+  const int item = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (item >= p.M * heads) return;
+  const int m = item / heads, h = item % heads;
+  const int d = EPL * 32, half = d / 2;
+  const size_t ldq = (size_t)heads * d;
+  const size_t pstride = (size_t)p.M * ldq;
+  const float* src = p.part + (size_t)m * ldq + (size_t)h * d + EPL * lane;
+  float x[EPL];
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) x[e] = src[e];
+  for (int s0 = 1; s0 < p.splits; s0 += 4) {
+    float y[4][EPL];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (s0 + u < p.splits)
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) y[u][e] = src[(size_t)(s0 + u) * pstride + e];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (s0 + u < p.splits)
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) x[e] += y[u][e];
+  }
+  if (h < p.nq + p.nkv) {
+    const T* w = static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane;
+    float ss = 0.f;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) ss += x[e] * x[e];
+    const float rstd = rsqrtf(warp_sum(ss) / (float)d + p.eps);
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) x[e] *= rstd * to_f(w[e]);
+    const int b = m / p.B, i = m % p.B;
+    const float* cs = p.rope + ((size_t)(b * p.B + i) * half + EPL * (lane & 15)) * 2;
+    const float sg = lane < 16 ? -1.f : 1.f;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+      const float partner = __shfl_xor_sync(0xffffffffu, x[e], 16);
+      x[e] = x[e] * cs[2 * e] + sg * partner * cs[2 * e + 1];
+    }
+  }
+  T* out = static_cast<T*>(p.out) + (size_t)m * ldq + (size_t)h * d + EPL * lane;
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) out[e] = from_f<T>(x[e]);
+}
+
+int launch_qkv_finalize(const QkvParams& p, int dtype, cudaStream_t s) {
+  const int items = p.M * (p.nq + 2 * p.nkv);
+  const dim3 grid((items + 7) / 8);
+  cudaError_t e;
+  if (p.d == 128)
+    e = dtype == LSP_DTYPE_BF16 ? launch_pdl(qkv_finalize_kernel<bf16, 4>, grid, dim3(256), 0, s, p)
+                                : launch_pdl(qkv_finalize_kernel<float, 4>, grid, dim3(256), 0, s, p);
+  else if (p.d == 64)
+    e = dtype == LSP_DTYPE_BF16 ? launch_pdl(qkv_finalize_kernel<bf16, 2>, grid, dim3(256), 0, s, p)
+                                : launch_pdl(qkv_finalize_kernel<float, 2>, grid, dim3(256), 0, s, p);
+  else
+    return LSP_ERR_SHAPE;
+  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 int attn_ksplit(int B, int W, int nq, int nkv) {

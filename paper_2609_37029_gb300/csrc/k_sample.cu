@@ -90,6 +90,8 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
   int* red_i = reinterpret_cast<int*>(red_v + kSampWarps * kMaxC);
   float* corr_s = reinterpret_cast<float*>(red_i + kSampWarps * kMaxC);   // [warps][C][17]
   T* e_s = reinterpret_cast<T*>(corr_s + kSampWarps * kMaxC * 17);        // [C8][lde]
+  // per-warp double buffer of the 16 W_c rows of the current / next tile (bf16 path)
+  bf16* wbuf = reinterpret_cast<bf16*>(e_s + (size_t)kMaxC * lde) + (size_t)(threadIdx.x >> 5) * 2 * 16 * lde;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   griddep_launch();
@@ -125,8 +127,8 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
 
   const T* Wc = static_cast<const T*>(p.Wc);
   const uint2 key = make_uint2((uint32_t)p.seed, (uint32_t)(p.seed >> 32));
-  const float temp = p.temperature;
-  const bool sample = temp > 0.f;
+  const bool sample = p.temperature > 0.f;
+  const float inv_temp = sample ? 1.0f / p.temperature : 1.0f;   // exact for T = 1
   float* cw = corr_s + (size_t)warp * kMaxC * 17;
   float bv[KG];
   int bi[KG];
@@ -141,28 +143,48 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
   };
   float4 zc[KG], zn[KG];
   int tile = blockIdx.x * kSampWarps + warp;
+  // the 16 W_c rows of a tile -> this warp's buffer `buf` (16-byte cp.async chunks)
+  auto stage_wc = [&](int t, int buf) {
+    if constexpr (sizeof(T) == 2) {
+      if (t < ntiles) {
+        const int chunks = 16 * rc / 8;
+        for (int c = lane; c < chunks; c += 32) {
+          const int r = c / (rc / 8), e = (c % (rc / 8)) * 8;
+          const bf16* src = reinterpret_cast<const bf16*>(Wc) + (size_t)(t * 16 + r) * rc + e;
+          bf16* dst = wbuf + (size_t)buf * 16 * lde + (size_t)r * lde + e;
+          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+        }
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+  };
+  stage_wc(tile, 0);
 #pragma unroll
   for (int k = 0; k < KG; ++k)
     if (tile < ntiles && lane + 32 * k < 4 * C) zc[k] = *reinterpret_cast<const float4*>(p.src + zoff(tile, k));
-  for (; tile < ntiles; tile += stride) {
+  int cur = 0;
+  for (; tile < ntiles; tile += stride, cur ^= 1) {
     const int next = tile + stride;
+    stage_wc(next, cur ^ 1);
 #pragma unroll
     for (int k = 0; k < KG; ++k)
       if (next < ntiles && lane + 32 * k < 4 * C) zn[k] = *reinterpret_cast<const float4*>(p.src + zoff(next, k));
     const int v0 = tile * 16;
     // correction W_c[v0:v0+16] . E_c(y)^T for all requests -> cw[b][v]
     if constexpr (sizeof(T) == 2) {
+      asm volatile("cp.async.wait_group 1;" ::: "memory");   // this tile's rows have landed
+      __syncwarp();
       const bf16* es = reinterpret_cast<const bf16*>(e_s);
-      const bf16* wr = reinterpret_cast<const bf16*>(Wc) + (size_t)(v0 + (lane >> 2)) * rc + (lane & 3) * 2;
+      const bf16* wr = wbuf + (size_t)cur * 16 * lde + (size_t)(lane >> 2) * lde + (lane & 3) * 2;
       float acc[KG][4];                                     // KG = ceil(C / 8) n-tiles of 8 requests
 #pragma unroll
       for (int nt = 0; nt < KG; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
       for (int kk = 0; kk < rc / 16; ++kk) {
         uint32_t a[4];
         a[0] = *reinterpret_cast<const uint32_t*>(wr + kk * 16);
-        a[1] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16);
+        a[1] = *reinterpret_cast<const uint32_t*>(wr + 8 * lde + kk * 16);
         a[2] = *reinterpret_cast<const uint32_t*>(wr + kk * 16 + 8);
-        a[3] = *reinterpret_cast<const uint32_t*>(wr + 8 * rc + kk * 16 + 8);
+        a[3] = *reinterpret_cast<const uint32_t*>(wr + 8 * lde + kk * 16 + 8);
 #pragma unroll
         for (int nt = 0; nt < KG; ++nt) {
           const bf16* er = es + (size_t)(nt * 8 + (lane >> 2)) * lde + (lane & 3) * 2 + kk * 16;
@@ -203,20 +225,21 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
         float sc[4] = {z.x, z.y, z.z, z.w};
         if (sample) {
           const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)step, (uint32_t)b, p.round), key);
-          sc[0] = sc[0] / temp + gumbel_of(x.x);
-          sc[1] = sc[1] / temp + gumbel_of(x.y);
-          sc[2] = sc[2] / temp + gumbel_of(x.z);
-          sc[3] = sc[3] / temp + gumbel_of(x.w);
+          sc[0] = sc[0] * inv_temp + gumbel_of(x.x);
+          sc[1] = sc[1] * inv_temp + gumbel_of(x.y);
+          sc[2] = sc[2] * inv_temp + gumbel_of(x.z);
+          sc[3] = sc[3] * inv_temp + gumbel_of(x.w);
         }
 #pragma unroll
         for (int e = 0; e < 4; ++e)
           if (better(sc[e], v + e, bv[k], bi[k])) { bv[k] = sc[e]; bi[k] = v + e; }
       }
     }
-    __syncwarp();
+    __syncwarp();                                           // wbuf[cur] is refilled next iteration
 #pragma unroll
     for (int k = 0; k < KG; ++k) zc[k] = zn[k];
   }
+  if constexpr (sizeof(T) == 2) asm volatile("cp.async.wait_all;" ::: "memory");
 
   // ---- per-CTA partial argmax of every request
 #pragma unroll
@@ -272,16 +295,18 @@ int sample_blocks(int num_sms) { return 2 * num_sms; }
 
 static size_t sample_smem(int rc, int es) {
   return kMaxC * sizeof(int) + 2 * kSampWarps * kMaxC * sizeof(float) +
-         (size_t)kSampWarps * kMaxC * 17 * sizeof(float) + (size_t)kMaxC * (rc + 8) * es;
+         (size_t)kSampWarps * kMaxC * 17 * sizeof(float) + (size_t)kMaxC * (rc + 8) * es +
+         (size_t)kSampWarps * 2 * 16 * (rc + 8) * 2;
 }
 
 template <typename T, int KG>
 static cudaError_t launch_step(const SampleParams& p, int step, size_t smem, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(sample_step_kernel<T, KG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)sample_smem(256, 4));
-    attr = true;
+  static size_t attr = 0;                 // largest dynamic shared memory granted so far
+  if (smem > attr) {
+    const cudaError_t e = cudaFuncSetAttribute(sample_step_kernel<T, KG>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = smem;
   }
   return launch_pdl(sample_step_kernel<T, KG>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step);
 }
@@ -290,6 +315,7 @@ int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
   const size_t smem = sample_smem(p.rc, es);
+  if (smem > 227 * 1024) return LSP_ERR_SHAPE;
 
   const int kg = (4 * p.C + 31) / 32;
   for (int step = 0; step < p.B; ++step) {

@@ -109,7 +109,15 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
     const int j = threadIdx.x + k * kRowThreads;
     if (j < h4) {
       float4 cv = ld4(c, j);
-      for (int s = 1; s < p.c_splits; ++s) cv = add4(cv, ld4(c + s * cstride, j));
+      for (int s0 = 1; s0 < p.c_splits; s0 += 4) {
+        float4 t[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (s0 + u < p.c_splits) t[u] = ld4(c + (s0 + u) * cstride, j);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (s0 + u < p.c_splits) cv = add4(cv, t[u]);
+      }
       xv[k] = add4(add4(ld4(src, j), ld4(pos, j)), cv);
       st4(p.x + (size_t)m * p.H, j, xv[k]);
       ss += dot4(xv[k]);
@@ -148,11 +156,20 @@ __global__ void __launch_bounds__(kRowThreads)
     const int j = threadIdx.x + k * kRowThreads;
     if (j < h4) xv[k] = ld4(row, j);
   }
-  for (int s = 0; s < splits; ++s) {
+  // splits in groups of four with all loads issued before the adds (in split order)
+  for (int s0 = 0; s0 < splits; s0 += 4) {
 #pragma unroll
     for (int k = 0; k < kMaxVec; ++k) {
       const int j = threadIdx.x + k * kRowThreads;
-      if (j < h4) xv[k] = add4(xv[k], ld4(prow + s * pstride, j));
+      if (j < h4) {
+        float4 t[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (s0 + u < splits) t[u] = ld4(prow + (s0 + u) * pstride, j);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (s0 + u < splits) xv[k] = add4(xv[k], t[u]);
+      }
     }
   }
 #pragma unroll

@@ -66,7 +66,7 @@ struct lsp_state {
   // workspace
   void* ws = nullptr;
   float *x = nullptr, *logits = nullptr, *rope = nullptr, *part = nullptr;
-  void *xn = nullptr, *o = nullptr, *act = nullptr;
+  void *xn = nullptr, *qkv = nullptr, *o = nullptr, *act = nullptr;
   size_t part_bytes = 0;
   float* part_val = nullptr;
   int* part_idx = nullptr;
@@ -214,6 +214,7 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   off = 0;
   const size_t w_x = off; off = align256(off + (size_t)M * c.H * 4);
   const size_t w_xn = off; off = align256(off + (size_t)M * c.H * es);
+  const size_t w_qkv = off; off = align256(off + (size_t)M * (c.nq + 2 * c.nkv) * c.d * es);
   const size_t w_o = off; off = align256(off + (size_t)M * c.nq * c.d * es);
   const size_t w_act = off; off = align256(off + (size_t)M * c.F * es);
   const size_t w_log = off; off = align256(off + (size_t)M * c.V * 4);
@@ -225,6 +226,7 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   char* w = static_cast<char*>(st->ws);
   st->x = reinterpret_cast<float*>(w + w_x);
   st->xn = w + w_xn;
+  st->qkv = w + w_qkv;
   st->o = w + w_o;
   st->act = w + w_act;
   st->logits = reinterpret_cast<float*>(w + w_log);
@@ -392,9 +394,14 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   for (int j = 0; j < c.D; ++j) {
     const lsp_layer_weights& lw = w->layer[j];
     if ((rc = gemm_launch(&st->qkv_op[j], s)) != LSP_OK) return rc;
+    QkvParams qp;
+    qp.part = st->part; qp.splits = st->qkv_op[j].p.splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
+    qp.rope = st->rope; qp.out = st->qkv; qp.M = M; qp.B = c.B; qp.nq = c.nq; qp.nkv = c.nkv; qp.d = c.d;
+    qp.eps = c.rms_eps;
+    if ((rc = launch_qkv_finalize(qp, c.dtype, s)) != LSP_OK) return rc;
     mark(st, ev++, s);
     AttnParams ap;
-    ap.qkv = st->part; ap.qkv_splits = st->qkv_op[j].p.splits; ap.q_norm = lw.q_norm; ap.k_norm = lw.k_norm; ap.rope = st->rope;
+    ap.qkv = st->qkv;
     ap.win_k = st->win_k; ap.win_v = st->win_v; ap.G = st->G; ap.m = st->m; ap.t = st->t;
     ap.out = st->o; ap.C = c.C; ap.B = c.B; ap.L = c.L; ap.nq = c.nq; ap.nkv = c.nkv; ap.d = c.d;
     ap.W = c.W; ap.R = c.R; ap.layer = c.layer_map[j]; ap.eps = c.rms_eps;

@@ -124,12 +124,22 @@ int launch_resid_norm(float* x, const float* part, int splits, const void* w, vo
                       int H, float eps, int dtype, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention
-struct AttnParams {
-  const float* qkv;       // [splits][M][(nq+2nkv)d] fp32 partial sums of the projections
-  int qkv_splits;
+// q | k | v of the block rows: sum of the projection's split-K partials, then
+// per-head RMSNorm (q_norm / k_norm) and rotary embedding on q and k.
+struct QkvParams {
+  const float* part;      // [splits][M][(nq+2nkv)d] fp32
+  int splits;
   const void* q_norm;     // [d]
   const void* k_norm;     // [d]
   const float* rope;      // [C][B][d/2][2]
+  void* out;              // [M][(nq+2nkv)d] dtype
+  int M, B, nq, nkv, d;
+  float eps;
+};
+int launch_qkv_finalize(const QkvParams& p, int dtype, cudaStream_t s);
+
+struct AttnParams {
+  const void* qkv;        // [M][(nq+2nkv)d] dtype: normalised, rotated q, k; v
   const void* win_k;      // state window of the tapped layer's base: [C][L][nkv][W][d]
   const void* win_v;
   const void* G;          // [L][nq][R][d]
