@@ -23,6 +23,7 @@ namespace lsp {
 constexpr int kSampThreads = 256;
 constexpr int kSampWarps = kSampThreads / 32;
 constexpr int kMaxC = 64;
+constexpr int kMaxPartialsPerLane = 16;    // sampler grids of up to 512 CTAs
 
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u;
@@ -64,11 +65,18 @@ __device__ __forceinline__ int resolve_prev(const SampleParams& p, int buf, int 
   int bi = 0x7fffffff;
   const float* pv = p.part_val + ((size_t)buf * p.C + b) * p.nblk;
   const int* pi = p.part_idx + ((size_t)buf * p.C + b) * p.nblk;
-  for (int gblk = lane; gblk < p.nblk; gblk += 32) {
-    const float v = pv[gblk];
-    const int i = pi[gblk];
-    if (better(v, i, bv, bi)) { bv = v; bi = i; }
+  // every load in flight before the first compare (nblk <= 32 * kMaxPartialsPerLane)
+  float v[kMaxPartialsPerLane];
+  int ix[kMaxPartialsPerLane];
+#pragma unroll
+  for (int k = 0; k < kMaxPartialsPerLane; ++k) {
+    const int g = lane + 32 * k;
+    v[k] = g < p.nblk ? pv[g] : -INFINITY;
+    ix[k] = g < p.nblk ? pi[g] : 0x7fffffff;
   }
+#pragma unroll
+  for (int k = 0; k < kMaxPartialsPerLane; ++k)
+    if (better(v[k], ix[k], bv, bi)) { bv = v[k]; bi = ix[k]; }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
@@ -291,7 +299,7 @@ __global__ void philox_words_kernel(uint64_t seed, uint32_t round, uint32_t b, u
   out[n] = w == 0 ? x.x : w == 1 ? x.y : w == 2 ? x.z : x.w;
 }
 
-int sample_blocks(int num_sms) { return 2 * num_sms; }
+int sample_blocks(int num_sms) { return std::min(2 * num_sms, 32 * kMaxPartialsPerLane); }
 
 static size_t sample_smem(int rc, int es) {
   return kMaxC * sizeof(int) + 2 * kSampWarps * kMaxC * sizeof(float) +
@@ -313,6 +321,7 @@ static cudaError_t launch_step(const SampleParams& p, int step, size_t smem, cud
 
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
+  if (p.nblk > 32 * kMaxPartialsPerLane) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
   const size_t smem = sample_smem(p.rc, es);
   if (smem > 227 * 1024) return LSP_ERR_SHAPE;
