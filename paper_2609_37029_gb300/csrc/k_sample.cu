@@ -5,14 +5,33 @@
 //     y_i = argmax_v (z_i[v] / T + g_{b,i,v})    (T > 0, Gumbel-max == sampling softmax(z_i / T))
 // with g = -log(-log u) from Philox4x32-10 (Salmon et al., SC'11).
 //
-// One launch per step i: every CTA first finishes step i-1's argmax from the
-// per-CTA partials (so y_{i-1} is known everywhere), gathers E_c(y_{i-1}) of
-// all C requests into shared memory, then sweeps its share of 16-row vocabulary
-// tiles: the correction W_c[v0:v0+16] E_c^T is one mma.sync tile per warp
-// (bf16 in, fp32 accumulate; fp32 storage uses FMA), the corrected logits are
-// read/written as float4, one Philox call feeds four vocabulary entries, and
-// a per-lane running argmax (ties to the lowest index) is reduced to one
-// partial per CTA and request.  A last tiny launch resolves y_B.
+// Two kernels compute the same thing.
+//
+// sample_persistent_kernel (bf16, C <= 16, rc in {32, 64}, vocabulary slice
+// fits shared memory): one cooperative launch for all B steps, one CTA per SM.
+// Each CTA owns a contiguous slice of 16-row vocabulary tiles and keeps its
+// W_c rows resident in shared memory for the whole launch.  Sixteen compute
+// warps form the correction as mma.sync tiles with the requests on M (16) and
+// the vocabulary on N, add the base logits (staged one step ahead by
+// cp.async), add the noise and keep a running argmax.  A control warp
+// publishes the CTA's best (value, index) of every request as one 64-bit
+// atomicMax key, arrives on the step's counter, waits (bounded) for every CTA,
+// reads y_i and gathers E_c(y_i) for the next step, while the compute warps
+// draw the next step's noise.  The k index of the contraction is permuted
+// identically in both operands so that each lane's operand words are
+// contiguous in shared memory, and the vocabulary columns are permuted so that
+// each lane's accumulators are four consecutive vocabulary entries (one
+// Philox call, one float4 of logits).
+//
+// sample_step_kernel (every other shape): one launch per step i: every CTA
+// first finishes step i-1's argmax from the per-CTA partials (so y_{i-1} is
+// known everywhere), gathers E_c(y_{i-1}) of all C requests into shared
+// memory, then sweeps its share of 16-row vocabulary tiles: the correction
+// W_c[v0:v0+16] E_c^T is one mma.sync tile per warp (bf16 in, fp32
+// accumulate; fp32 storage uses FMA), the corrected logits are read/written
+// as float4, one Philox call feeds four vocabulary entries, and a per-lane
+// running argmax (ties to the lowest index) is reduced to one partial per CTA
+// and request.  A last tiny launch resolves y_B.
 #include <algorithm>
 
 #include "common.cuh"
@@ -279,6 +298,338 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
   }
 }
 
+// ------------------------------------------------------------------ persistent kernel
+constexpr int kPWarps = 16;                          // compute warps
+constexpr int kPThreads = (kPWarps + 1) * 32;        // + the control warp
+constexpr int kPTilesPerWarp = 4;
+constexpr int kPMaxTiles = kPWarps * kPTilesPerWarp; // 64 tiles = 1024 vocabulary rows per CTA
+constexpr int kPMaxC = 16;
+constexpr int kSlotStride = 16;                      // u64 words between step keys: one 128-byte line
+                                                     // per (step, request) spreads the atomics over L2
+constexpr int kBarKeys = 1;                          // compute warps -> control warp: keys ready
+constexpr int kBarNext = 2;                          // control warp -> compute warps: E_c(y_i) ready
+
+// Order-preserving 64-bit key of (value, index): a larger value wins, equal
+// values go to the lower index; -0 ranks as +0.
+__device__ __forceinline__ unsigned long long arg_key(float v, int i) {
+  uint32_t u = __float_as_uint(v);
+  if (u == 0x80000000u) u = 0u;
+  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ((unsigned long long)u << 32) | (uint32_t)~(uint32_t)i;
+}
+
+__device__ __forceinline__ unsigned long long max_u64(unsigned long long a, unsigned long long b) {
+  return a > b ? a : b;
+}
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void named_arrive(int id, int count) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// Wait (every lane of a warp, same address) until *c >= target; false after kWaitLimitNs.
+__device__ __forceinline__ bool wait_count(const unsigned* c, unsigned target) {
+  if (ld_acquire_u32(c) >= target) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (ld_acquire_u32(c) >= target) return true;
+    if ((i & 63u) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
+  }
+}
+
+// Control warp: E_c rows of the current tokens (lane r < C holds y_r) into Es,
+// 16-byte chunk c of row r stored at chunk c ^ (r & 1).
+template <int CH>
+__device__ __forceinline__ void gather_e(const bf16* Ec, int y, int C, int rc, uint8_t* Es, int lane) {
+#pragma unroll
+  for (int i0 = 0; i0 < kPMaxC * CH; i0 += 32) {
+    const int i = i0 + lane, r = i / CH, c = i % CH;
+    const int yr = __shfl_sync(0xffffffffu, y, r);
+    if (r < C) {
+      const uint4 v = *reinterpret_cast<const uint4*>(Ec + (size_t)yr * rc + c * 8);
+      *reinterpret_cast<uint4*>(Es + r * (CH * 16) + ((c ^ (r & 1)) * 16)) = v;
+    }
+  }
+}
+
+// KS = rc / 16 k-steps of the m16n8k16 contraction.
+template <int KS>
+__global__ void __launch_bounds__(kPThreads, 1)
+    sample_persistent_kernel(const SampleParams p, const int ntiles) {
+  constexpr int RB = KS * 32;        // bytes of one W_c / E_c row
+  constexpr int CH = RB / 16;        // 16-byte chunks per row
+  constexpr int TCH = KS / 2;        // chunks of one lane's k range
+  extern __shared__ __align__(128) uint8_t psm[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nblk = gridDim.x;
+  const int t_begin = (int)(((long long)blockIdx.x * ntiles) / nblk);
+  const int cnt = (int)(((long long)(blockIdx.x + 1) * ntiles) / nblk) - t_begin;
+  const int tpc = (ntiles + nblk - 1) / nblk;
+  uint8_t* Ws = psm;                                                    // [tpc*16][RB]
+  float4* Zs = reinterpret_cast<float4*>(psm + (size_t)tpc * 16 * RB);  // [tpc][2][32]
+  uint8_t* Es = reinterpret_cast<uint8_t*>(Zs + (size_t)tpc * 64);      // [16][RB]
+  unsigned long long* red = reinterpret_cast<unsigned long long*>(Es + kPMaxC * RB);   // [warps][16]
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(red + kPWarps * kPMaxC);
+  unsigned long long* slots = p.sync;                                   // [B][16][kSlotStride]
+  unsigned* counts = reinterpret_cast<unsigned*>(p.sync + (size_t)p.B * kPMaxC * kSlotStride);   // [B]
+  const bf16* Wc = static_cast<const bf16*>(p.Wc);
+  const bf16* Ec = static_cast<const bf16*>(p.Ec);
+  const int C = p.C, B = p.B, V = p.V, rc = p.rc;
+  const bool sample = p.temperature > 0.f;
+  const float inv_temp = sample ? 1.0f / p.temperature : 1.0f;
+  const uint2 key = make_uint2((uint32_t)p.seed, (uint32_t)(p.seed >> 32));
+  const int g = lane >> 2, q = lane & 3;                               // mma group / thread in group
+
+  // ---- prologue: W_c slice, zero E rows, step-0 logits, y_0, E_c(y_0)
+  for (int i = tid; i < cnt * 16 * CH; i += kPThreads) {
+    const int r = i / CH, c = i % CH;
+    cp_async16(Ws + r * RB + ((c ^ (r & 1)) * 16), Wc + (size_t)(t_begin * 16 + r) * rc + c * 8, 16);
+  }
+  for (int i = tid; i < kPMaxC * RB / 16; i += kPThreads)
+    reinterpret_cast<uint4*>(Es)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (tid == 0) *abort_flag = 0;
+  // E_c rows are gathered at random every step: keep the table in L2 (this CTA's share)
+  if (tid == kPWarps * 32) {
+    const size_t bytes = (size_t)V * rc * 2;
+    const size_t share = (bytes / nblk + 4095) / 4096 * 4096;
+    const size_t lo = share * blockIdx.x, hi = lo + share < bytes ? lo + share : bytes;
+    const uint64_t pol = policy_evict_last();
+    for (size_t o = lo; o < hi; o += 4096) {
+      const uint32_t n = (uint32_t)(hi - o < 4096 ? hi - o : 4096);
+      asm volatile("cp.async.bulk.prefetch.L2.global.L2::cache_hint [%0], %1, %2;" ::"l"(
+                       reinterpret_cast<const char*>(Ec) + o),
+                   "r"(n), "l"(pol)
+                   : "memory");
+    }
+  }
+
+  auto issue_z = [&](int s) {        // this lane's own logits of step s (same lane reads them)
+#pragma unroll
+    for (int j = 0; j < kPTilesPerWarp; ++j) {
+      const int lt = warp + kPWarps * j;
+      if (lt < cnt) {
+        const int v = (t_begin + lt) * 16 + 4 * q;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int r = g + 8 * h;
+          const bool ok = r < C;
+          cp_async16(&Zs[(lt * 2 + h) * 32 + lane], p.src + (ok ? ((size_t)r * B + s) * V + v : 0),
+                     ok ? 16u : 0u);
+        }
+      }
+    }
+  };
+  float gn[kPTilesPerWarp][2][4];      // noise of the step about to be scored
+  auto draw_noise = [&](int s) {
+#pragma unroll
+    for (int j = 0; j < kPTilesPerWarp; ++j) {
+      const int lt = warp + kPWarps * j;
+      if (lt < cnt) {
+        const int v = (t_begin + lt) * 16 + 4 * q;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const uint4 x = philox4x32_10(
+              make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(g + 8 * h), p.round), key);
+          gn[j][h][0] = gumbel_of(x.x);
+          gn[j][h][1] = gumbel_of(x.y);
+          gn[j][h][2] = gumbel_of(x.z);
+          gn[j][h][3] = gumbel_of(x.w);
+        }
+      }
+    }
+  };
+
+  int y = 0;                                                            // control warp: y of lane < C
+  if (warp < kPWarps) {
+    issue_z(0);
+  } else {
+    __syncwarp();
+    if (lane < C) {
+      y = p.prev[(size_t)lane * p.prev_stride];
+      if (y < 0 || y >= V) {
+        if (blockIdx.x == 0) set_err(p.err, LSP_DEV_BAD_TOKEN);
+        y = 0;
+      }
+    }
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  __syncthreads();                                                      // E rows zeroed
+  if (warp == kPWarps) gather_e<CH>(Ec, y, C, rc, Es, lane);
+  if (warp < kPWarps && sample) draw_noise(0);
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();                                                      // W_c slice and E_c(y_0) visible
+
+  if (warp < kPWarps) {
+    // ================= compute warps
+    for (int s = 0; s < B; ++s) {
+      // A operand: E_c(y) rows g and g + 8 over this lane's k range
+      uint32_t a[KS][4];
+      {
+        uint32_t e0[2 * KS], e1[2 * KS];
+#pragma unroll
+        for (int c = 0; c < TCH; ++c) {
+          const int pc = (TCH * q + c) ^ (g & 1);
+          const uint4 u0 = *reinterpret_cast<const uint4*>(Es + g * RB + pc * 16);
+          const uint4 u1 = *reinterpret_cast<const uint4*>(Es + (g + 8) * RB + pc * 16);
+          e0[4 * c] = u0.x; e0[4 * c + 1] = u0.y; e0[4 * c + 2] = u0.z; e0[4 * c + 3] = u0.w;
+          e1[4 * c] = u1.x; e1[4 * c + 1] = u1.y; e1[4 * c + 2] = u1.z; e1[4 * c + 3] = u1.w;
+        }
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+          a[ks][0] = e0[2 * ks];
+          a[ks][1] = e1[2 * ks];
+          a[ks][2] = e0[2 * ks + 1];
+          a[ks][3] = e1[2 * ks + 1];
+        }
+      }
+      asm volatile("cp.async.wait_all;" ::: "memory");                  // this lane's z_s landed
+      const int v_first = (t_begin + warp) * 16 + 4 * q;
+      float bv[2] = {-INFINITY, -INFINITY};
+      int bi[2] = {v_first, v_first};
+#pragma unroll
+      for (int j = 0; j < kPTilesPerWarp; ++j) {
+        const int lt = warp + kPWarps * j;
+        if (lt >= cnt) break;                                           // warp-uniform
+        const int v = (t_begin + lt) * 16 + 4 * q;
+        float acc[2][4];
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+          // column n = g of n-tile t is vocabulary row 4 (g >> 1) + 2 t + (g & 1) of the tile
+          const int row = lt * 16 + 4 * (g >> 1) + 2 * t + (g & 1);
+          uint32_t bw[2 * KS];
+#pragma unroll
+          for (int c = 0; c < TCH; ++c) {
+            const uint4 u = *reinterpret_cast<const uint4*>(Ws + row * RB + (((TCH * q + c) ^ (g & 1)) * 16));
+            bw[4 * c] = u.x; bw[4 * c + 1] = u.y; bw[4 * c + 2] = u.z; bw[4 * c + 3] = u.w;
+          }
+          acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
+#pragma unroll
+          for (int ks = 0; ks < KS; ++ks) mma_bf16_s(acc[t], a[ks], bw[2 * ks], bw[2 * ks + 1]);
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const float4 z = Zs[(lt * 2 + h) * 32 + lane];
+          float zc[4] = {z.x + acc[0][2 * h], z.y + acc[0][2 * h + 1], z.z + acc[1][2 * h],
+                         z.w + acc[1][2 * h + 1]};
+          // corrected logits go out after the keys are published (below)
+          if (p.dst) Zs[(lt * 2 + h) * 32 + lane] = make_float4(zc[0], zc[1], zc[2], zc[3]);
+          if (sample) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) zc[e] = zc[e] * inv_temp + gn[j][h][e];
+          }
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if (zc[e] > bv[h]) { bv[h] = zc[e]; bi[h] = v + e; }
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        unsigned long long k = warp < cnt ? arg_key(bv[h], bi[h]) : 0ull;
+        k = max_u64(k, __shfl_xor_sync(0xffffffffu, k, 1));
+        k = max_u64(k, __shfl_xor_sync(0xffffffffu, k, 2));
+        if (q == 0) red[warp * kPMaxC + g + 8 * h] = k;
+      }
+      named_arrive(kBarKeys, kPThreads);
+      // HBM traffic of this lane (corrected logits out, next logits in) and the
+      // next step's noise overlap the grid-wide wait
+      if (p.dst) {
+#pragma unroll
+        for (int j = 0; j < kPTilesPerWarp; ++j) {
+          const int lt = warp + kPWarps * j;
+          if (lt < cnt) {
+            const int v = (t_begin + lt) * 16 + 4 * q;
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              if (g + 8 * h < C)
+                *reinterpret_cast<float4*>(p.dst + ((size_t)(g + 8 * h) * B + s) * V + v) =
+                    Zs[(lt * 2 + h) * 32 + lane];
+          }
+        }
+      }
+      if (s + 1 == B) break;
+      issue_z(s + 1);                                                   // slots already consumed
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      if (sample) draw_noise(s + 1);
+      named_bar(kBarNext, kPThreads);
+      if (*abort_flag) break;
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    return;
+  }
+
+  // ================= control warp
+  const size_t zrow = (size_t)cnt * 16 * sizeof(float);                  // this CTA's slice of one logits row
+  for (int s = 0; s < B; ++s) {
+    // pull the next step's logits slice into L2 while the compute warps score this one
+    if (s + 1 < B && lane < C && zrow > 0)
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
+                       p.src + ((size_t)lane * B + s + 1) * V + (size_t)t_begin * 16),
+                   "r"((uint32_t)zrow)
+                   : "memory");
+    named_bar(kBarKeys, kPThreads);
+    if (lane < C) {
+      unsigned long long k = 0ull;
+#pragma unroll
+      for (int w = 0; w < kPWarps; ++w) k = max_u64(k, red[w * kPMaxC + lane]);
+      atomicMax(&slots[(s * kPMaxC + lane) * kSlotStride], k);
+    }
+    __syncwarp();
+    if (lane == 0) red_release_add(&counts[s], 1u);                     // orders the warp's key atomics
+    const bool last = s + 1 == B;
+    if (last && blockIdx.x != 0) return;                                // only CTA 0 needs y_B
+    const bool ok = __all_sync(0xffffffffu, wait_count(&counts[s], (unsigned)nblk));
+    if (!ok) {
+      if (lane == 0) set_err(p.err, LSP_DEV_TIMEOUT);
+      if (!last) {
+        if (lane == 0) *abort_flag = 1;
+        __syncwarp();
+        named_arrive(kBarNext, kPThreads);
+      }
+      return;
+    }
+    if (lane < C) {
+      y = (int)~(uint32_t)ld_relaxed_u64(&slots[(s * kPMaxC + lane) * kSlotStride]);
+      if (y < 0 || y >= V) {                                            // no key arrived: corrupt sync words
+        set_err(p.err, LSP_DEV_TIMEOUT);
+        y = 0;
+      }
+      if (blockIdx.x == 0) p.out_tokens[(size_t)lane * B + s] = y;
+    }
+    if (last) {
+      // every CTA has arrived on every counter, so no one reads the sync words
+      // again: leave them zero for the next launch
+      __syncwarp();
+      for (int i = lane; i < B * kPMaxC; i += 32) slots[i * kSlotStride] = 0ull;
+      for (int i = lane; i < B; i += 32) counts[i] = 0u;
+      return;
+    }
+    gather_e<CH>(Ec, y, C, rc, Es, lane);
+    __syncwarp();
+    named_arrive(kBarNext, kPThreads);
+  }
+}
+
 __global__ void __launch_bounds__(kSampThreads) sample_final_kernel(const SampleParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   griddep_launch();
@@ -319,8 +670,75 @@ static cudaError_t launch_step(const SampleParams& p, int step, size_t smem, cud
   return launch_pdl(sample_step_kernel<T, KG>, dim3(p.nblk), dim3(kSampThreads), smem, s, p, step);
 }
 
+size_t sample_sync_bytes(int B) {
+  return ((size_t)B * kPMaxC * kSlotStride * sizeof(unsigned long long) + (size_t)B * sizeof(unsigned) +
+          255) / 256 * 256;
+}
+
+static size_t persistent_smem(int tpc, int rc) {
+  const size_t rb = (size_t)rc * 2;
+  return (size_t)tpc * 16 * rb + (size_t)tpc * 64 * 16 + kPMaxC * rb +
+         (size_t)kPWarps * kPMaxC * sizeof(unsigned long long) + 16;
+}
+
+template <int KS>
+static int launch_persistent(const SampleParams& p, cudaStream_t s) {
+  const int ntiles = p.V / 16;
+  const int nblk = std::min(p.num_sms, ntiles);
+  const int tpc = (ntiles + nblk - 1) / nblk;
+  if (tpc > kPMaxTiles) return LSP_ERR_SHAPE;
+  const size_t smem = persistent_smem(tpc, p.rc);
+  if (smem > 227 * 1024) return LSP_ERR_SHAPE;
+  static size_t attr = 0;
+  if (smem > attr) {
+    if (cudaFuncSetAttribute(sample_persistent_kernel<KS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess)
+      return LSP_ERR_CUDA;
+    attr = smem;
+  }
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sample_persistent_kernel<KS>, kPThreads,
+                                                    smem) != cudaSuccess)
+    return LSP_ERR_CUDA;
+  if (per_sm < 1) return LSP_ERR_SHAPE;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(nblk);
+  cfg.blockDim = dim3(kPThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr_c[1];
+  attr_c[0].id = cudaLaunchAttributeCooperative;       // every CTA resident: the step waits are safe
+  attr_c[0].val.cooperative = 1;
+  cfg.attrs = attr_c;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sample_persistent_kernel<KS>, p, ntiles) == cudaSuccess ? LSP_OK
+                                                                                          : LSP_ERR_CUDA;
+}
+
+// The persistent kernel's shape limits (anything else takes the per-step kernel).
+static bool persistent_ok(const SampleParams& p, int dtype) {
+  if (dtype != LSP_DTYPE_BF16 || p.C > kPMaxC || (p.rc != 32 && p.rc != 64) || !p.sync || p.num_sms < 1)
+    return false;
+  const int ntiles = p.V / 16;
+  const int nblk = std::min(p.num_sms, ntiles);
+  const int tpc = (ntiles + nblk - 1) / nblk;
+  if (tpc > kPMaxTiles || persistent_smem(tpc, p.rc) > 227 * 1024) return false;
+  int dev = 0, coop = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess)
+    return false;
+  return coop != 0;
+}
+
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
+  // float4 / 16-byte accesses to the logits and the correction tables
+  if ((reinterpret_cast<uintptr_t>(p.src) | reinterpret_cast<uintptr_t>(p.dst) |
+       reinterpret_cast<uintptr_t>(p.Ec) | reinterpret_cast<uintptr_t>(p.Wc)) & 15)
+    return LSP_ERR_ARG;
+  if (persistent_ok(p, dtype))
+    return p.rc == 32 ? launch_persistent<2>(p, s) : launch_persistent<4>(p, s);
+
   if (p.nblk > 32 * kMaxPartialsPerLane) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
   const size_t smem = sample_smem(p.rc, es);

@@ -6,9 +6,12 @@
 // section, a process whose device memory is fully reserved by another
 // framework's caching allocator, or code that must not create a state object
 // (lsp_state_create allocates the interface and a workspace).  The sampler's
-// only scratch is the per-CTA argmax partials of two consecutive steps, so this
-// variant keeps them in a fixed file-scope __device__ array instead.  Every GPU
-// that loads the library holds that array until the process exits.
+// only scratch is the per-CTA argmax partials of two consecutive steps and the
+// per-step keys and arrival counters of the persistent kernel, so this variant
+// keeps them in a fixed file-scope __device__ array instead.  Every GPU that
+// loads the library holds that array until the process exits.  The counters
+// are cleared on the caller's stream before every launch, so a launch that
+// gave up waiting cannot affect the next one.
 #include <cmath>
 #include <mutex>
 
@@ -71,7 +74,11 @@ extern "C" int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_
   if (rc_setup != LSP_OK) return rc_setup;
   const int nblk = lsp::sample_blocks(ds->num_sms);
   const size_t part = (size_t)2 * nblk * C;                  // values, then indices
-  if (part * (sizeof(float) + sizeof(int)) > kStaticScratchBytes) return LSP_ERR_SHAPE;
+  const size_t sync_off = (part * (sizeof(float) + sizeof(int)) + 255) / 256 * 256;
+  const size_t sync_bytes = lsp::sample_sync_bytes(B);
+  if (sync_off + sync_bytes > kStaticScratchBytes) return LSP_ERR_SHAPE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ds->ptr + sync_off, 0, sync_bytes, s) != cudaSuccess) return LSP_ERR_CUDA;
   lsp::SampleParams p;
   p.src = base_logits;
   p.dst = out_logits;
@@ -82,14 +89,16 @@ extern "C" int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_
   p.out_tokens = out_tokens;
   p.part_val = reinterpret_cast<float*>(ds->ptr);
   p.part_idx = reinterpret_cast<int*>(ds->ptr + part * sizeof(float));
+  p.sync = reinterpret_cast<unsigned long long*>(ds->ptr + sync_off);
   p.err = reinterpret_cast<unsigned*>(dev_error);
   p.C = C;
   p.B = B;
   p.V = V;
   p.rc = rc;
   p.nblk = nblk;
+  p.num_sms = ds->num_sms;
   p.temperature = sp->temperature;
   p.round = sp->round;
   p.seed = sp->seed;
-  return lsp::launch_sample(p, dtype, static_cast<cudaStream_t>(stream));
+  return lsp::launch_sample(p, dtype, s);
 }

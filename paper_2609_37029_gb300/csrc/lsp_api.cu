@@ -70,6 +70,8 @@ struct lsp_state {
   size_t part_bytes = 0;
   float* part_val = nullptr;
   int* part_idx = nullptr;
+  unsigned long long* sample_sync = nullptr;
+  size_t sample_sync_bytes = 0;
   int nblk = 0;
   // cached projection plans
   bool have_plans = false;
@@ -222,6 +224,7 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   const size_t w_part = off; off = align256(off + pbytes);
   const size_t w_pv = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
   const size_t w_pi = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
+  const size_t w_sync = off; off = align256(off + sample_sync_bytes(c.B));
   if (cudaMalloc(&st->ws, off) != cudaSuccess) { free_state(st); return LSP_ERR_NOMEM; }
   char* w = static_cast<char*>(st->ws);
   st->x = reinterpret_cast<float*>(w + w_x);
@@ -235,6 +238,8 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   st->part_bytes = pbytes;
   st->part_val = reinterpret_cast<float*>(w + w_pv);
   st->part_idx = reinterpret_cast<int*>(w + w_pi);
+  st->sample_sync = reinterpret_cast<unsigned long long*>(w + w_sync);
+  st->sample_sync_bytes = sample_sync_bytes(c.B);
   if (cudaMemset(st->ws, 0, off) != cudaSuccess || cudaMemset(st->base, 0, o_done + l.done) != cudaSuccess) {
     free_state(st);
     return LSP_ERR_CUDA;
@@ -356,8 +361,9 @@ static int run_sampler(lsp_state* st, const float* src, float* dst, const int32_
   const lsp_config& c = st->cfg;
   SampleParams p;
   p.src = src; p.dst = dst; p.prev = prev; p.prev_stride = prev_stride; p.Ec = Ec; p.Wc = Wc;
-  p.out_tokens = out_tokens; p.part_val = st->part_val; p.part_idx = st->part_idx; p.err = st->err;
-  p.C = c.C; p.B = c.B; p.V = c.V; p.rc = c.rc; p.nblk = st->nblk;
+  p.out_tokens = out_tokens; p.part_val = st->part_val; p.part_idx = st->part_idx;
+  p.sync = st->sample_sync; p.err = st->err;
+  p.C = c.C; p.B = c.B; p.V = c.V; p.rc = c.rc; p.nblk = st->nblk; p.num_sms = st->num_sms;
   p.temperature = sp->temperature; p.round = sp->round; p.seed = sp->seed;
   return launch_sample(p, c.dtype, s);
 }
@@ -506,6 +512,10 @@ int lsp_get_error(lsp_state* st, uint32_t* dev_error, int clear, lsp_stream_t st
       cudaStreamSynchronize(s) != cudaSuccess)
     return LSP_ERR_CUDA;
   if (clear && v && cudaMemsetAsync(st->err, 0, sizeof(unsigned), s) != cudaSuccess) return LSP_ERR_CUDA;
+  // a sampler launch that gave up waiting leaves its step counters behind
+  if (clear && (v & LSP_DEV_TIMEOUT) &&
+      cudaMemsetAsync(st->sample_sync, 0, st->sample_sync_bytes, s) != cudaSuccess)
+    return LSP_ERR_CUDA;
   *dev_error = v;
   if (v & LSP_DEV_TIMEOUT) return LSP_ERR_TIMEOUT;
   return v ? LSP_ERR_STATE : LSP_OK;

@@ -160,15 +160,19 @@ struct SampleParams {
   const void* Ec;
   const void* Wc;
   int32_t* out_tokens;    // [C][B]
-  float* part_val;        // [2][nblk][C]
+  float* part_val;        // [2][nblk][C]   (per-step kernel)
   int* part_idx;          // [2][nblk][C]
+  unsigned long long* sync;   // sample_sync_bytes(B): step keys + arrival counts (persistent
+                              // kernel); all zero between launches
   unsigned* err;
   int C, B, V, rc, nblk;
+  int num_sms;
   float temperature;
   uint32_t round;
   uint64_t seed;
 };
 int sample_blocks(int num_sms);
+size_t sample_sync_bytes(int B);
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s);
 int launch_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint32_t* out,
                         int count, cudaStream_t s);

@@ -158,9 +158,10 @@ SAMP = synth.LspShape("samp", C=5, B=16, L=1, D=1, H=128, nq=1, nkv=1, d=128, F=
 
 
 @pytest.mark.parametrize("temperature", [0.0, 1.0, 0.7])
-@pytest.mark.parametrize("dt", ["bf16", "f32"])
-def test_sampler_matches_oracle(lsp, temperature, dt):
-    s = SAMP if dt == "bf16" else SAMP.with_(dtype="f32", d=64, nq=2, nkv=2)
+@pytest.mark.parametrize("dt,C", [("bf16", 5), ("bf16", 16), ("bf16", 20), ("f32", 5)])
+def test_sampler_matches_oracle(lsp, temperature, dt, C):
+    # bf16 with C <= 16 runs the persistent single-launch kernel, the rest the per-step kernel
+    s = SAMP.with_(C=C) if dt == "bf16" else SAMP.with_(dtype="f32", d=64, nq=2, nkv=2)
     st = lsp.lsp_state_create(lsp.make_config(s))
     try:
         g = torch.Generator().manual_seed(11)
@@ -172,9 +173,16 @@ def test_sampler_matches_oracle(lsp, temperature, dt):
         toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
         zout = torch.zeros(s.C, s.B, s.V, device="cuda")
         sp = lsp.make_sample_params(temperature, seed=0x1234ABCD5678, rnd=9)
-        lsp.lsp_sample(st, z0.cuda(), prev.cuda(), Ec.cuda(), Wc.cuda(), sp, toks, zout)
+        args = (z0.cuda(), prev.cuda(), Ec.cuda(), Wc.cuda())
+        lsp.lsp_sample(st, *args, sp, toks, zout)
         torch.cuda.synchronize()
         toks_g, z_g = toks.cpu().numpy(), f64(zout)
+        # a second launch on the same state reproduces the first bit for bit
+        toks2 = torch.zeros_like(toks)
+        zout2 = torch.zeros_like(zout)
+        lsp.lsp_sample(st, *args, sp, toks2, zout2)
+        torch.cuda.synchronize()
+        assert torch.equal(toks2, toks) and torch.equal(zout2, zout)
         checked = 0
         for b in range(s.C):
             t_o, z_o, marg = oracle.sample_block(f64(z0[b]), int(prev[b]), f64(Ec), f64(Wc), temperature,
