@@ -10,8 +10,11 @@
 //               activation tile per stage into an S-deep mbarrier ring, plus
 //               L2 prefetches of the weight tiles `pd` stages ahead
 //   warp 1      TMEM allocation and the single-thread tcgen05.mma issue
-//   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulators and a fused
-//               store (fp32, storage dtype, SwiGLU) or a split-K partial
+//   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulators, the fused
+//               output (fp32, storage dtype, SwiGLU, or a split-K partial)
+//               staged in shared memory 16-32 tokens at a time and written
+//               by TMA tensor stores (double-buffered), so the global writes
+//               are full-line bulk copies that overlap the next chunk
 //
 // Launched as a programmatic dependent: before the preceding kernel finishes,
 // the producer already streams this launch's weights (L2 prefetch and the
@@ -91,11 +94,82 @@ __device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int sp
   }
 }
 
+constexpr uint32_t kXchgStride = 33;                          // SwiGLU exchange row (floats)
+constexpr uint32_t kXchgBytes = 17408;                        // 128 x 33 floats, 1 KB aligned
+
+// Epilogue through shared memory and TMA stores (4 warps, r = accumulator
+// row = output feature of the tile).  Chunk c of TT tokens: every thread
+// loads its row's TT accumulators, writes them (or, for SwiGLU, the
+// activation of its share after a gate/up exchange) into staging buffer
+// c & 1, and one thread stores the buffer with a TMA tensor store into the
+// [split][token][feature] view of Y.  Token rows past M and feature columns
+// past N fall outside the view and are not written.
+template <typename T>
+__device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensorMap* to, uint8_t* smem,
+                                             uint32_t lane_base, int ntl, int tile0, int split,
+                                             int r) {
+  const bool swiglu = p.mode == EPI_SWIGLU;
+  const bool f32out = p.mode == EPI_F32 || p.mode == EPI_PARTIAL;
+  const int es = f32out ? 4 : (int)sizeof(T);
+  const int cols = swiglu ? 64 : kTileRows;                   // output features of one weight tile
+  const int TT = p.out_tok;
+  float* xchg = reinterpret_cast<float*>(smem);              // SwiGLU: [128][kXchgStride]
+  uint8_t* stg0 = smem + (swiglu ? kXchgBytes : 0);
+  const uint32_t buf_bytes = (uint32_t)(TT * cols * es);     // <= 16 KB
+  const bool issuer = r == 0;
+  int chunk = 0;
+  for (int w = 0; w < ntl; ++w) {
+    for (int m0 = 0; m0 < p.m_pad; m0 += TT, ++chunk) {
+      float v[32];
+      const uint32_t col = (uint32_t)(w * p.m_pad + m0);
+      if (TT == 32) tmem_ld32(lane_base + col, v);
+      else tmem_ld16(lane_base + col, v);
+      uint8_t* stg = stg0 + (chunk & 1) * buf_bytes;
+      if (issuer && chunk >= 2) bulk_wait_read<1>();         // the store two chunks back has read stg
+      named_bar(1, 128);
+      if (swiglu) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < TT) xchg[r * kXchgStride + j] = v[j];
+        named_bar(1, 128);
+        // thread (f = r & 63, half = r >> 6) forms tokens [half * TT/2, (half + 1) * TT/2)
+        const int f = r & 63, t0 = (r >> 6) * (TT / 2);
+        T* o = reinterpret_cast<T*>(stg);
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if (j < TT / 2) {
+            const int t = t0 + j;
+            const float g = xchg[f * kXchgStride + t];
+            const float u = xchg[(f + 64) * kXchgStride + t];
+            o[t * 64 + f] = from_f<T>(g / (1.0f + expf(-g)) * u);
+          }
+      } else if (f32out) {
+        float* o = reinterpret_cast<float*>(stg);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < TT) o[j * kTileRows + r] = v[j];
+      } else {
+        T* o = reinterpret_cast<T*>(stg);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < TT) o[j * kTileRows + r] = from_f<T>(v[j]);
+      }
+      fence_proxy_async_smem();
+      named_bar(1, 128);
+      if (issuer) {
+        tma_store_3d(to, smem_u32(stg), (tile0 + w) * cols, m0, split);
+        bulk_commit();
+      }
+    }
+  }
+  if (issuer) bulk_wait_read<0>();                            // staging smem is released at exit
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap ta0, const __grid_constant__ CUtensorMap ta1,
                 const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb,
-                const GemmParams p) {
+                const __grid_constant__ CUtensorMap to, const __grid_constant__ GemmParams p) {
   using G = GemmType<T>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -132,6 +206,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     fence_barrier_init();
     tma_prefetch_desc(&ta0);
     tma_prefetch_desc(&tb);
+    if (p.tma_out) tma_prefetch_desc(&to);
   }
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), (uint32_t)p.tmem_cols);
   tc_fence_before();
@@ -145,15 +220,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ------------------------------------------------------------ TMA producer
     const uint64_t pol_w = policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
-    // weight tile w of this CTA: tensor map and first row
-    auto a_src = [&](int w, const CUtensorMap** ta, int* row) {
+    // weight tile w of this CTA: segment (tensor map) and first row within it
+    auto a_seg = [&](int w) {
       const int tile = tile0 + w;
-      int seg = 0;
-      if (p.nseg > 2 && tile >= p.seg_tile0[2]) seg = 2;
-      else if (p.nseg > 1 && tile >= p.seg_tile0[1]) seg = 1;
-      *ta = seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2);
-      *row = (tile - p.seg_tile0[seg]) * kTileRows;
+      return (p.nseg > 2 && tile >= p.seg_tile0[2]) ? 2 : (p.nseg > 1 && tile >= p.seg_tile0[1]) ? 1 : 0;
     };
+    auto a_map = [&](int seg) { return seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2); };
     auto load_a = [&](int i, uint32_t sa, uint32_t bar) {
       const int kx = (kb0 + i) * G::BK;
       for (int w = 0; w < ntl; ++w) {
@@ -162,10 +234,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tma_load_2d(sa + w * kTileBytes, &ta0, bar, kx, row, pol_w);
           tma_load_2d(sa + w * kTileBytes + 64 * 128, &ta1, bar, kx, row, pol_w);
         } else {
-          const CUtensorMap* ta;
-          int row;
-          a_src(w, &ta, &row);
-          tma_load_2d(sa + w * kTileBytes, ta, bar, kx, row, pol_w);
+          const int seg = a_seg(w);
+          tma_load_2d(sa + w * kTileBytes, a_map(seg), bar, kx, (tile0 + w - p.seg_tile0[seg]) * kTileRows,
+                      pol_w);
         }
       }
     };
@@ -176,10 +247,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tma_prefetch_l2(&ta0, kx, (tile0 + w) * 64);
           tma_prefetch_l2(&ta1, kx, (tile0 + w) * 64);
         } else {
-          const CUtensorMap* ta;
-          int row;
-          a_src(w, &ta, &row);
-          tma_prefetch_l2(ta, kx, row);
+          const int seg = a_seg(w);
+          tma_prefetch_l2(a_map(seg), kx, (tile0 + w - p.seg_tile0[seg]) * kTileRows);
         }
       }
     };
@@ -249,8 +318,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (!ok) *s_abort = 1;
     tc_fence_after();
     named_bar(1, 128);
-    if (*s_abort == 0) {
-      const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
+    const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
+    if (*s_abort == 0 && p.tma_out) {
+      epilogue_tma<T>(p, &to, smem, lane_base, ntl, tile0, split, r);
+    } else if (*s_abort == 0) {
       for (int w = 0; w < ntl; ++w)
         for (int tt = 0; tt < p.n_tok_tiles; ++tt)
           for (int c0 = 0; c0 < p.bn; c0 += 16) {
@@ -318,6 +389,25 @@ static int make_map(CUtensorMap* m, int dtype, const void* ptr, int K, int rows,
                    2, const_cast<void*>(ptr), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? LSP_OK : LSP_ERR_CUDA;
+}
+
+// [splits][M][N] view of the output (row stride ldy) for TMA stores of
+// box (cols features, tok tokens, 1 split); no swizzle.
+static int make_out_map(CUtensorMap* m, bool f32, const void* Y, int N, int M, int splits, int ldy,
+                        int cols, int tok) {
+  auto enc = encoder();
+  if (!enc) return LSP_ERR_UNSUPPORTED;
+  const int es = f32 ? 4 : 2;
+  if (((uintptr_t)Y & 15) || ((size_t)ldy * es) % 16) return LSP_ERR_SHAPE;
+  cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)splits};
+  cuuint64_t strides[2] = {(cuuint64_t)ldy * es, (cuuint64_t)M * ldy * es};
+  cuuint32_t box[3] = {(cuuint32_t)cols, (cuuint32_t)tok, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                   const_cast<void*>(Y), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? LSP_OK : LSP_ERR_CUDA;
 }
 
@@ -461,6 +551,15 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     if ((rc = make_map(&op->a[i], dtype, W[si], K, seg_rows[si], box_rows)) != LSP_OK) return rc;
   }
   if ((rc = make_map(&op->b, dtype, X, K, M, p.bn)) != LSP_OK) return rc;
+  // TMA-store epilogue when the output view can be described (else per-thread stores)
+  p.out_tok = (p.m_pad % 32) ? 16 : 32;
+  {
+    const bool f32 = mode == EPI_F32 || mode == EPI_PARTIAL || dtype == LSP_DTYPE_F32;
+    const int cols = mode == EPI_SWIGLU ? 64 : kTileRows;
+    p.tma_out = make_out_map(&op->out, f32, Y, p.N, M, splits, ldy, cols, p.out_tok) == LSP_OK &&
+                std::getenv("LSP_GEMM_SCALAR_EPI") == nullptr;
+    if (!p.tma_out) op->out = op->b;       // unused placeholder
+  }
   op->grid = dim3((unsigned)n_ctas, (unsigned)splits, 1);
   op->smem = (size_t)p.stages * stage_bytes + 1024 + 256;
   return LSP_OK;
@@ -473,7 +572,7 @@ static int launch_t(const GemmOp* op, cudaStream_t s) {
     cudaFuncSetAttribute(gemm_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
   });
   const cudaError_t e = launch_pdl(gemm_kernel<T>, op->grid, dim3(kGemmThreads), op->smem, s,
-                                   op->a[0], op->a[1], op->a[2], op->b, op->p);
+                                   op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 

@@ -49,6 +49,8 @@ struct GemmParams {
   int seg_tile0[3];     // first tile index of each A segment
   int nseg;
   int bn, n_tok_tiles, m_pad, stages, tmem_cols, pd;
+  int tma_out;          // 1: the epilogue stages tiles in shared memory and TMA-stores them
+  int out_tok;          // tokens per staged output chunk (16 or 32)
   void* Y;
   int ldy;
   unsigned* err;
@@ -57,6 +59,7 @@ struct GemmParams {
 struct GemmOp {
   CUtensorMap a[3];
   CUtensorMap b;
+  CUtensorMap out;      // [splits][M][N] view of Y for the TMA-store epilogue
   GemmParams p;
   int dtype;
   dim3 grid;
