@@ -454,9 +454,12 @@ static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
 // Split-K factor from a cost model in units of one k-block of one of two
 // co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
 // fixed per-CTA cost) + the consumer's re-read of the fp32 split partials
-// from L2 (partial_cost per split).  A lone CTA on an SM streams a k-block in
-// ~0.63 of that time.
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok) {
+// from L2 (partial_cost per split).  With a small token tile a lone CTA on an
+// SM streams a k-block in ~0.63 of that time; with a wide one (>= 128 tokens)
+// a lone CTA is no faster: its single MMA issuer keeps the tensor pipe only
+// partly busy, and a second CTA on the SM hides that.
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok,
+                     bool wide) {
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(16, kblocks); ++s) {
@@ -464,7 +467,7 @@ int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, 
     const bool two = two_ok && ctas * 4 >= (long long)num_sms * 5;
     const long long slots = two ? 2LL * num_sms : num_sms;
     const long long waves = (ctas + slots - 1) / slots;
-    const double per = (double)((kblocks + s - 1) / s) * (two ? 1.0 : 0.63) + 2.0;
+    const double per = (double)((kblocks + s - 1) / s) * (two || wide ? 1.0 : 0.63) + 2.0;
     const double cost = (double)waves * per + (s > 1 ? partial_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
@@ -486,7 +489,7 @@ void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, in
   if (*splits <= 0)
     *splits = mode == EPI_PARTIAL
                   ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows),
-                                     two_per_sm_fits(*wt, m_pad))
+                                     two_per_sm_fits(*wt, m_pad), m_pad >= 128)
                   : 1;
   *splits = std::max(1, std::min(*splits, kblocks));
 }

@@ -11,7 +11,9 @@
 // resid_norm_kernel: x += sum of a projection's split-K partials (the
 // residual add of the o and down projections, in split order), then
 // x / sqrt(mean(x^2) + eps) * w (Qwen3 RMSNorm) into the storage dtype that
-// the next projection's TMA reads.
+// the next projection's TMA reads; one CTA of up to 1024 threads per row.
+#include <algorithm>
+
 #include "common.cuh"
 #include "lsp_internal.h"
 
@@ -137,8 +139,13 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kRowThreads)
+// One CTA per token row with (up to) one 16-byte vector per thread: every
+// partial load of a thread is in flight at once and 32 warps per row keep the
+// SM busy while they land.
+constexpr int kNormThreads = 1024;
+
+template <typename T, int VPT>
+__global__ void __launch_bounds__(kNormThreads)
     resid_norm_kernel(float* __restrict__ x, const float* __restrict__ part, int splits,
                       const T* __restrict__ w, T* __restrict__ out, int M, int H, float eps) {
   __shared__ float red[32];
@@ -149,32 +156,32 @@ __global__ void __launch_bounds__(kRowThreads)
   const float* prow = part + (size_t)m * H;
   const size_t pstride = (size_t)M * H;
   const int h4 = H / 4;
-  float4 xv[kMaxVec];
+  float4 xv[VPT];
   float ss = 0.f;
 #pragma unroll
-  for (int k = 0; k < kMaxVec; ++k) {
-    const int j = threadIdx.x + k * kRowThreads;
+  for (int k = 0; k < VPT; ++k) {
+    const int j = threadIdx.x + k * blockDim.x;
     if (j < h4) xv[k] = ld4(row, j);
   }
-  // splits in groups of four with all loads issued before the adds (in split order)
-  for (int s0 = 0; s0 < splits; s0 += 4) {
+  // splits in groups of eight with all loads issued before the adds (in split order)
+  for (int s0 = 0; s0 < splits; s0 += 8) {
 #pragma unroll
-    for (int k = 0; k < kMaxVec; ++k) {
-      const int j = threadIdx.x + k * kRowThreads;
+    for (int k = 0; k < VPT; ++k) {
+      const int j = threadIdx.x + k * blockDim.x;
       if (j < h4) {
-        float4 t[4];
+        float4 t[8];
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+        for (int u = 0; u < 8; ++u)
           if (s0 + u < splits) t[u] = ld4(prow + (s0 + u) * pstride, j);
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+        for (int u = 0; u < 8; ++u)
           if (s0 + u < splits) xv[k] = add4(xv[k], t[u]);
       }
     }
   }
 #pragma unroll
-  for (int k = 0; k < kMaxVec; ++k) {
-    const int j = threadIdx.x + k * kRowThreads;
+  for (int k = 0; k < VPT; ++k) {
+    const int j = threadIdx.x + k * blockDim.x;
     if (j < h4) {
       if (splits > 0) st4(row, j, xv[k]);
       ss += dot4(xv[k]);
@@ -182,8 +189,8 @@ __global__ void __launch_bounds__(kRowThreads)
   }
   const float rstd = rsqrtf(block_sum(ss, red) / (float)H + eps);
 #pragma unroll
-  for (int k = 0; k < kMaxVec; ++k) {
-    const int j = threadIdx.x + k * kRowThreads;
+  for (int k = 0; k < VPT; ++k) {
+    const int j = threadIdx.x + k * blockDim.x;
     if (j < h4) {
       const float4 wv = ld4(w, j);
       st4(out + (size_t)m * H, j, make_float4(xv[k].x * rstd * wv.x, xv[k].y * rstd * wv.y,
@@ -201,16 +208,27 @@ int launch_combine(const CombineParams& p, int dtype, cudaStream_t s) {
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
+template <typename T>
+static cudaError_t launch_norm_t(float* x, const float* part, int splits, const void* w, void* out, int M,
+                                 int H, float eps, cudaStream_t s) {
+  const int h4 = H / 4;
+  const int threads = std::min(kNormThreads, (h4 + 31) / 32 * 32);
+  const int vpt = (h4 + threads - 1) / threads;
+  const T* wt = static_cast<const T*>(w);
+  T* ot = static_cast<T*>(out);
+  switch (vpt) {
+    case 1: return launch_pdl(resid_norm_kernel<T, 1>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
+    case 2: return launch_pdl(resid_norm_kernel<T, 2>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
                       int H, float eps, int dtype, cudaStream_t s) {
-  if (H > kRowThreads * kMaxPerThread) return LSP_ERR_SHAPE;
-  cudaError_t e;
-  if (dtype == LSP_DTYPE_BF16)
-    e = launch_pdl(resid_norm_kernel<bf16>, dim3(M), dim3(kRowThreads), 0, s, x, part, splits,
-                   static_cast<const bf16*>(w), static_cast<bf16*>(out), M, H, eps);
-  else
-    e = launch_pdl(resid_norm_kernel<float>, dim3(M), dim3(kRowThreads), 0, s, x, part, splits,
-                   static_cast<const float*>(w), static_cast<float*>(out), M, H, eps);
+  if (H > 2 * 4 * kNormThreads || H % 4) return LSP_ERR_SHAPE;
+  const cudaError_t e = dtype == LSP_DTYPE_BF16
+                            ? launch_norm_t<bf16>(x, part, splits, w, out, M, H, eps, s)
+                            : launch_norm_t<float>(x, part, splits, w, out, M, H, eps, s);
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 

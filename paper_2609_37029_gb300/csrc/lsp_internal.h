@@ -77,7 +77,8 @@ int gemm_launch(const GemmOp* op, cudaStream_t s);
 // The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 = choose).
 void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok);
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok,
+                     bool wide);
 double gemm_partial_cost(int M, int N);
 int gemm_kblocks(int K, int dtype);
 // Deterministic sum of `splits` fp32 partials [splits][n] into y[n].
