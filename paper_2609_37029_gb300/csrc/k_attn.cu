@@ -16,6 +16,8 @@
 // (bf16 in, fp32 accumulate), and the key splits merge through shared memory.
 // attn_simple_kernel (fp32 storage): plain FMA version, one CTA per
 // (request, query head), for the fp32 reference shape.
+#include <type_traits>
+
 #include "common.cuh"
 #include "lsp_internal.h"
 
@@ -73,7 +75,11 @@ static AttnLayout attn_layout(int B, int W, int nq, int nkv, int ksplit) {
   a.bytes = a.off_vs + (size_t)a.rep * 16 * row;
   return a;
 }
-static size_t attn_merge_bytes(int nwarps) { return (size_t)nwarps * (16 * kHD + 32) * sizeof(float); }
+// Key-split merge scratch per warp: o[16][kOs] (padded: conflict-free float2
+// stores of the mma accumulator layout) then max[16] and sum[16].
+constexpr int kOs = kHD + 8;
+constexpr int kMergeRec = 16 * kOs + 32;
+static size_t attn_merge_bytes(int nwarps) { return (size_t)nwarps * kMergeRec * sizeof(float); }
 
 __global__ void __launch_bounds__(512)
     attn_mma_kernel(const AttnParams p, const int rep, const int ksplit, const int rows_bw) {
@@ -247,16 +253,14 @@ __global__ void __launch_bounds__(512)
   // ---- merge the key splits of each head (scratch reuses the K/V staging area)
   __syncthreads();
   float* scratch = reinterpret_cast<float*>(sKbw);
-  float* so = scratch + (size_t)warp * (16 * kHD + 32);
-  float* sml = so + 16 * kHD;
+  float* so = scratch + (size_t)warp * kMergeRec;
+  float* sml = so + 16 * kOs;
   const int r0 = lane >> 2;
 #pragma unroll
   for (int n = 0; n < 16; ++n) {
     const int col = n * 8 + (lane & 3) * 2;
-    so[r0 * kHD + col] = o[n][0];
-    so[r0 * kHD + col + 1] = o[n][1];
-    so[(r0 + 8) * kHD + col] = o[n][2];
-    so[(r0 + 8) * kHD + col + 1] = o[n][3];
+    *reinterpret_cast<float2*>(so + r0 * kOs + col) = make_float2(o[n][0], o[n][1]);
+    *reinterpret_cast<float2*>(so + (r0 + 8) * kOs + col) = make_float2(o[n][2], o[n][3]);
   }
   if ((lane & 3) == 0) {
     sml[r0] = rmax[0];
@@ -267,21 +271,29 @@ __global__ void __launch_bounds__(512)
   __syncthreads();
   bf16* out = static_cast<bf16*>(p.out);
   const int ldo = p.nq * kHD;
-  for (int idx = tid; idx < rep * B * kHD; idx += nthr) {
-    const int e = idx % kHD, i = (idx / kHD) % B, h2 = idx / (kHD * B);
+  // thread -> (head h2, query i, 4 columns e..e+3)
+  for (int idx = tid; idx < rep * B * (kHD / 4); idx += nthr) {
+    const int e = (idx % (kHD / 4)) * 4, i = (idx / (kHD / 4)) % B, h2 = idx / ((kHD / 4) * B);
+    const float* base = scratch + (size_t)h2 * ksplit * kMergeRec;
     float M = -INFINITY;
+    for (int k = 0; k < ksplit; ++k) M = fmaxf(M, base[(size_t)k * kMergeRec + 16 * kOs + i]);
+    float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+    float den = 0.f;
     for (int k = 0; k < ksplit; ++k) {
-      const float* ml = scratch + (size_t)(h2 * ksplit + k) * (16 * kHD + 32) + 16 * kHD;
-      M = fmaxf(M, ml[i]);
+      const float* sw = base + (size_t)k * kMergeRec;
+      const float f = exp2f((sw[16 * kOs + i] - M) * sl2);
+      den += f * sw[16 * kOs + 16 + i];
+      const float4 v = *reinterpret_cast<const float4*>(sw + i * kOs + e);
+      num.x += f * v.x;
+      num.y += f * v.y;
+      num.z += f * v.z;
+      num.w += f * v.w;
     }
-    float num = 0.f, den = 0.f;
-    for (int k = 0; k < ksplit; ++k) {
-      const float* sw = scratch + (size_t)(h2 * ksplit + k) * (16 * kHD + 32);
-      const float f = exp2f((sw[16 * kHD + i] - M) * sl2);
-      den += f * sw[16 * kHD + 16 + i];
-      num += f * sw[i * kHD + e];
-    }
-    out[(size_t)(b * B + i) * ldo + (size_t)(g * rep + h2) * kHD + e] = __float2bfloat16_rn(num / den);
+    const float inv = 1.0f / den;
+    uint2 wv;
+    wv.x = pack_bf16(num.x * inv, num.y * inv);
+    wv.y = pack_bf16(num.z * inv, num.w * inv);
+    *reinterpret_cast<uint2*>(out + (size_t)(b * B + i) * ldo + (size_t)(g * rep + h2) * kHD + e) = wv;
   }
 }
 
@@ -381,21 +393,28 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
   const size_t ldq = (size_t)heads * d;
   const size_t pstride = (size_t)p.M * ldq;
   const float* src = p.part + (size_t)m * ldq + (size_t)h * d + EPL * lane;
+  // the lane's EPL consecutive values of every split as one vector load each,
+  // all in flight before the adds (which run in split order)
+  using V = typename std::conditional<EPL == 4, float4, float2>::type;
   float x[EPL];
+  {
+    const V v0 = *reinterpret_cast<const V*>(src);
+    const float* f0 = reinterpret_cast<const float*>(&v0);
 #pragma unroll
-  for (int e = 0; e < EPL; ++e) x[e] = src[e];
-  for (int s0 = 1; s0 < p.splits; s0 += 4) {
-    float y[4][EPL];
+    for (int e = 0; e < EPL; ++e) x[e] = f0[e];
+  }
+  for (int s0 = 1; s0 < p.splits; s0 += 8) {
+    V y[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (s0 + u < p.splits)
+    for (int u = 0; u < 8; ++u)
+      if (s0 + u < p.splits) y[u] = *reinterpret_cast<const V*>(src + (size_t)(s0 + u) * pstride);
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) y[u][e] = src[(size_t)(s0 + u) * pstride + e];
+    for (int u = 0; u < 8; ++u)
+      if (s0 + u < p.splits) {
+        const float* f = reinterpret_cast<const float*>(&y[u]);
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (s0 + u < p.splits)
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) x[e] += y[u][e];
+        for (int e = 0; e < EPL; ++e) x[e] += f[e];
+      }
   }
   if (h < p.nq + p.nkv) {
     const T* w = static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane;

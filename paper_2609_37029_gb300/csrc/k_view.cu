@@ -24,6 +24,36 @@ constexpr int kViewThreads = 256;
 constexpr int kViewWarps = kViewThreads / 32;
 constexpr int kViewChunk = 32;       // new rows staged per pass (one per lane)
 
+// N (2 or 4) consecutive fp32 / bf16 values <-> registers with one vector access
+template <int N>
+__device__ __forceinline__ void load_vec(const float* p, float* v) {
+  if constexpr (N == 4) {
+    const float4 x = *reinterpret_cast<const float4*>(p);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+  } else {
+    const float2 x = *reinterpret_cast<const float2*>(p);
+    v[0] = x.x; v[1] = x.y;
+  }
+}
+template <int N>
+__device__ __forceinline__ void load_vec(const bf16* p, float* v) {
+  if constexpr (N == 4) {
+    const uint2 r = *reinterpret_cast<const uint2*>(p);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
+    v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+  } else {
+    const uint32_t r = *reinterpret_cast<const uint32_t*>(p);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r));
+    v[0] = a.x; v[1] = a.y;
+  }
+}
+template <int N>
+__device__ __forceinline__ void store_vec(float* p, const float* v) {
+  if constexpr (N == 4) *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  else *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+}
+
 template <typename T, int DPL, int QPW>
 __global__ void __launch_bounds__(kViewThreads)
     view_update_kernel(const ViewParams p) {
@@ -64,10 +94,9 @@ __global__ void __launch_bounds__(kViewThreads)
     for (int e = 0; e < DPL; ++e) { ma[i][e] = 0.f; gq[i][e] = 0.f; }
     if (q < Q) {
       eta_a[i] = p.eta[qbase + q];
-      const float* mrow = p.m + (qbase + q) * d + lane * DPL;
-      const T* grow = Gp + (gbase + q) * d + lane * DPL;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) { ma[i][e] = mrow[e]; gq[i][e] = to_f(grow[e]); }
+      // the lane's DPL consecutive entries as one vector load each
+      load_vec<DPL>(p.m + (qbase + q) * d + lane * DPL, ma[i]);
+      load_vec<DPL>(Gp + (gbase + q) * d + lane * DPL, gq[i]);
     }
   }
   const float scale = rsqrtf((float)d);
@@ -110,6 +139,7 @@ __global__ void __launch_bounds__(kViewThreads)
       if (q >= Q) continue;                                            // warp-uniform
       // scores of this query over the chunk: lane j keeps s_j
       float s_mine = -INFINITY;
+#pragma unroll 4
       for (int j = 0; j < nrows; ++j) {
         const float* kr = sK + j * d + lane * DPL;
         float part = 0.f;
@@ -126,6 +156,7 @@ __global__ void __launch_bounds__(kViewThreads)
       float mn[DPL];
 #pragma unroll
       for (int e = 0; e < DPL; ++e) mn[e] = 0.f;
+#pragma unroll 4
       for (int j = 0; j < nrows; ++j) {
         const float pj = __shfl_sync(0xffffffffu, e_mine, j);
         const float* vr = sV + j * d + lane * DPL;
@@ -149,9 +180,7 @@ __global__ void __launch_bounds__(kViewThreads)
   for (int i = 0; i < QPW; ++i) {
     const int q = warp + i * kViewWarps;
     if (q < Q) {
-      float* mrow = p.m + (qbase + q) * d + lane * DPL;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) mrow[e] = ma[i][e];
+      store_vec<DPL>(p.m + (qbase + q) * d + lane * DPL, ma[i]);
       if (lane == 0) p.eta[qbase + q] = eta_a[i];
     }
   }
