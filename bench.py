@@ -190,10 +190,6 @@ def round_work(s, mean_delta):
     return nb, fl
 
 
-def launches_per_round(s):
-    return 1 + 1 + 1 + 7 * s.D + 1 + (s.B + 1)
-
-
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -549,7 +545,7 @@ def run_ours(args, dist):
            "stages_us": {k: round(v, 2) for k, v in stages.items()},
            "e2e": {"value": dist.world * s.C * s.B / (e2e_ms * 1e-3), "unit": UNIT,
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-           "gpu_launches": launches_per_round(s) * args.steps,
+           "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
            "clocks": clocks, "sweep": sweep, "cpu_baseline": cpu}
     if dist.rank == 0:
         print(json.dumps(out), flush=True)

@@ -269,6 +269,10 @@ int lsp_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i,
  * n_events must be 0 (off) or lsp_stage_count(st) + 1.  Event records are
  * capturable, so a captured round carries them as graph nodes. */
 int lsp_stage_count(lsp_state* st);
+/* Number of kernel launches one round (lsp_view_update + lsp_draft) issues
+ * for this state's config on the current device (the sampler is one launch
+ * or B + 1 depending on the shape); 0 for a null state. */
+int lsp_round_launches(lsp_state* st);
 const char* lsp_stage_name(lsp_state* st, int k);
 int lsp_set_stage_events(lsp_state* st, void* const* events, int n_events);
 

@@ -730,6 +730,8 @@ static bool persistent_ok(const SampleParams& p, int dtype) {
   return coop != 0;
 }
 
+int sample_launches(const SampleParams& p, int dtype) { return persistent_ok(p, dtype) ? 1 : p.B + 1; }
+
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
   // float4 / 16-byte accesses to the logits and the correction tables

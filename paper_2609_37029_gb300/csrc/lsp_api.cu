@@ -481,6 +481,16 @@ int lsp_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint
 
 int lsp_stage_count(lsp_state* st) { return st ? stage_total(st->cfg) : 0; }
 
+int lsp_round_launches(lsp_state* st) {
+  if (!st) return 0;
+  const lsp_config& c = st->cfg;
+  SampleParams p = {};
+  p.C = c.C; p.B = c.B; p.V = c.V; p.rc = c.rc; p.num_sms = st->num_sms; p.sync = st->sample_sync;
+  // view update, fuse, combine; per layer q/k/v GEMM + finalize, attention, o, norm, gate/up, down,
+  // norm; LM head; the sampler
+  return 3 + 8 * c.D + 1 + sample_launches(p, c.dtype);
+}
+
 const char* lsp_stage_name(lsp_state* st, int k) {
   if (!st || k < 0 || k >= stage_total(st->cfg)) return nullptr;
   if (k == 0) return "view_update";

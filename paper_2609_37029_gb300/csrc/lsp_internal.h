@@ -178,6 +178,8 @@ struct SampleParams {
 int sample_blocks(int num_sms);
 size_t sample_sync_bytes(int B);
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s);
+// Kernel launches one launch_sample call issues for these shapes on this device.
+int sample_launches(const SampleParams& p, int dtype);
 int launch_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i, uint32_t* out,
                         int count, cudaStream_t s);
 

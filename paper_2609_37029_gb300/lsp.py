@@ -91,6 +91,7 @@ _f = {
                              c_void_p, c_int, c_void_p),
     "lsp_get_error": _sig("lsp_get_error", c_int, c_void_p, POINTER(c_uint32), c_int, c_void_p),
     "lsp_stage_count": _sig("lsp_stage_count", c_int, c_void_p),
+    "lsp_round_launches": _sig("lsp_round_launches", c_int, c_void_p),
     "lsp_stage_name": _sig("lsp_stage_name", c_char_p, c_void_p, c_int),
     "lsp_set_stage_events": _sig("lsp_set_stage_events", c_int, c_void_p, POINTER(c_void_p), c_int),
     "lsp_state_export": _sig("lsp_state_export", c_int, c_void_p, c_void_p, c_size_t, c_void_p),
@@ -224,6 +225,10 @@ def lsp_get_error(st, clear=True, stream=None):
     bits = c_uint32(0)
     rc = _f["lsp_get_error"](st, ctypes.byref(bits), 1 if clear else 0, _stream(stream))
     return rc, bits.value
+
+
+def lsp_round_launches(st) -> int:
+    return _f["lsp_round_launches"](st)
 
 
 def lsp_stage_count(st) -> int:
