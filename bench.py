@@ -222,6 +222,33 @@ def profiled_traffic(kernel_file, workload):
         return None
 
 
+def prefill_leg(wl, rows, hbm, dist, reps=5):
+    """lsp_prefill of one request's `rows`-row prefix: device time, K/V bytes read, HBM fraction."""
+    s, lsp = wl.s, wl.lsp
+    s1 = s.with_(C=1)
+    k, v, h = synth.make_features(s1, rows, seed=wl.seed_base + 9000, device="cuda")
+    st = wl.new_state()
+    for _ in range(2):
+        lsp.lsp_prefill(st, 0, k[0], v[0], h[0])
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dist.barrier()
+    e0.record()
+    for _ in range(reps):
+        lsp.lsp_prefill(st, 0, k[0], v[0], h[0])
+    e1.record()
+    torch.cuda.synchronize()
+    us = dist.max(e0.elapsed_time(e1) * 1e3 / reps)
+    kv = 2 * s.L * rows * s.nkv * s.d * 2
+    flops = 2 * 2 * s.L * s.nq * s.R * rows * s.d           # G K^T and P V
+    lsp.lsp_state_destroy(st)
+    del k, v, h
+    return {"rows": rows, "us_per_request": us, "kv_bytes": kv, "achieved_gbs": kv / us * 1e-3,
+            "frac_hbm": kv / us * 1e-3 / hbm, "flops": flops,
+            "note": "mma.sync score and value products (P V as bf16 high + remainder): "
+                    "tensor-issue bound on the legacy path, not HBM"}
+
+
 # ------------------------------------------------------------------ workload
 class Workload:
     def __init__(self, s, lsp, seed_base):
@@ -530,6 +557,11 @@ def run_ours(args, dist):
                  "state_bytes": lsp.lsp_state_bytes(wl.cfg), "state_bytes_constant": True}
         lsp.lsp_state_destroy(st2)
 
+    # prefill (the one O(t) drafter step): one request's whole prefix at the largest sweep length
+    prefill = None
+    if prefixes and not args.no_sweep and s.dtype == "bf16":
+        prefill = prefill_leg(wl, max(prefixes), hbm, dist)
+
     cpu = None
     if want_cpu:
         leg = oracle_leg(wl, kept, args.cpu_budget)
@@ -546,7 +578,7 @@ def run_ours(args, dist):
            "e2e": {"value": dist.world * s.C * s.B / (e2e_ms * 1e-3), "unit": UNIT,
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
            "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
-           "clocks": clocks, "sweep": sweep, "cpu_baseline": cpu}
+           "clocks": clocks, "sweep": sweep, "prefill": prefill, "cpu_baseline": cpu}
     if dist.rank == 0:
         print(json.dumps(out), flush=True)
     lsp.lsp_state_destroy(st)

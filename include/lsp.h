@@ -241,6 +241,21 @@ int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, cons
                        const lsp_sample_params* sp, int32_t* out_tokens, float* out_logits,
                        uint32_t* dev_error, lsp_stream_t stream);
 
+/* Prefill (Sec. 2.2, Eq. global-summary, App. A.2; Fig. 3: the summary is
+ * initialised over the full prefix during target prefill): replace request
+ * b's interface by the one its whole prefix of t = f->rows rows defines --
+ * summary (eta, m) = attention of the R summary queries of every tapped layer
+ * and query head over all t rows, window ring = the last min(t, W) rows
+ * (prefix row p in slot p mod W), boundary = hidden state of row t-1, and t.
+ *   f->k, f->v: device dtype [L][t][nkv][d] (request b only); f->h: device
+ *   dtype [L][t][H]; borrowed for the call's duration on `stream`.
+ * Equivalent to folding the t rows into an empty request with
+ * lsp_view_update, but split over the whole GPU (segments of the prefix
+ * merged in order with Eq. summary-update; deterministic).  Needs an
+ * initialised state (G); bf16 storage with d = 128, R <= 16, nq/nkv <= 8 (else
+ * LSP_ERR_UNSUPPORTED: use lsp_view_update).  Other requests are untouched. */
+int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream);
+
 /* Dense projection Y = X W^T with the drafter's tensor-core GEMM (the kernel
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].

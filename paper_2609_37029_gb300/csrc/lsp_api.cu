@@ -70,6 +70,7 @@ struct lsp_state {
   size_t part_bytes = 0;
   float* part_val = nullptr;
   int* part_idx = nullptr;
+  float* prefill_ws = nullptr;       // prefill segment partials (bf16, d = 128 configs)
   unsigned long long* sample_sync = nullptr;
   size_t sample_sync_bytes = 0;
   int nblk = 0;
@@ -225,6 +226,8 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   const size_t w_pv = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
   const size_t w_pi = off; off = align256(off + (size_t)2 * st->nblk * c.C * 4);
   const size_t w_sync = off; off = align256(off + sample_sync_bytes(c.B));
+  const bool prefill_ok = c.dtype == LSP_DTYPE_BF16 && c.d == 128;
+  const size_t w_pf = off; off = align256(off + (prefill_ok ? prefill_ws_floats(c.L, c.nq) * sizeof(float) : 0));
   if (cudaMalloc(&st->ws, off) != cudaSuccess) { free_state(st); return LSP_ERR_NOMEM; }
   char* w = static_cast<char*>(st->ws);
   st->x = reinterpret_cast<float*>(w + w_x);
@@ -239,6 +242,7 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   st->part_val = reinterpret_cast<float*>(w + w_pv);
   st->part_idx = reinterpret_cast<int*>(w + w_pi);
   st->sample_sync = reinterpret_cast<unsigned long long*>(w + w_sync);
+  st->prefill_ws = prefill_ok ? reinterpret_cast<float*>(w + w_pf) : nullptr;
   st->sample_sync_bytes = sample_sync_bytes(c.B);
   if (cudaMemset(st->ws, 0, off) != cudaSuccess || cudaMemset(st->base, 0, o_done + l.done) != cudaSuccess) {
     free_state(st);
@@ -298,6 +302,19 @@ int lsp_view_update(lsp_state* st, const lsp_target_feats* f, const int32_t* acc
   const int rc = launch_view_update(p, c.dtype, S(stream));
   mark(st, 1, S(stream));
   return rc;
+}
+
+int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream) {
+  if (!st || !f || !f->k || !f->v || !f->h || f->rows < 1) return LSP_ERR_ARG;
+  if (!st->initialized) return LSP_ERR_STATE;
+  const lsp_config& c = st->cfg;
+  if (b < 0 || b >= c.C) return LSP_ERR_ARG;
+  PrefillParams p;
+  p.k = f->k; p.v = f->v; p.hid = f->h; p.rows = f->rows; p.G = st->G;
+  p.win_k = st->win_k; p.win_v = st->win_v; p.m = st->m; p.eta = st->eta; p.h = st->h; p.t = st->t;
+  p.ws = st->prefill_ws;
+  p.b = b; p.L = c.L; p.nq = c.nq; p.nkv = c.nkv; p.d = c.d; p.W = c.W; p.R = c.R; p.H = c.H;
+  return launch_prefill(p, c.dtype, S(stream));
 }
 
 static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {

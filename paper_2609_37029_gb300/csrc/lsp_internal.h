@@ -155,6 +155,26 @@ struct AttnParams {
 };
 int launch_attention(const AttnParams& p, int dtype, cudaStream_t s);
 
+// ------------------------------------------------------------------ prefill
+struct PrefillParams {
+  const void* k;          // request b's prefix K: [L][rows][nkv][d] dtype
+  const void* v;          // V, same layout
+  const void* hid;        // hidden states [L][rows][H] dtype
+  int rows;               // t (>= 1)
+  const void* G;          // [L][nq][R][d]
+  void* win_k;            // state window [C][L][nkv][W][d]
+  void* win_v;
+  float* m;               // [C][L][nq][R][d]
+  float* eta;             // [C][L][nq][R]
+  void* h;                // [C][L][H]
+  int64_t* t;             // [C]
+  float* ws;              // prefill_ws_floats(L, nq) segment partials
+  int b, L, nq, nkv, d, W, R, H;
+};
+constexpr int kPrefillMaxSeg = 64;   // prefix segments (CTAs per tapped layer x KV head)
+size_t prefill_ws_floats(int L, int nq);
+int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s);
+
 // ------------------------------------------------------------------ sampler
 struct SampleParams {
   const float* src;       // [C][B][V] base logits
