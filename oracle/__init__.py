@@ -14,6 +14,8 @@ written from the paper's text in its own order and notation:
 * sampler.py -- the low-rank Markov correction (Eq. markov) and sequential
                 proposal sampling (Eq. proposal-factorization) with Gumbel-max
                 over a Philox4x32-10 stream.
+* verify.py  -- target-side verification of a drafted block (Eq. acceptance,
+                Eq. residual, the bonus draw of Sec. 2.1).
 * philox.py  -- Philox4x32-10 (Salmon et al., SC'11) from its published definition.
 
 Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may import
@@ -21,7 +23,8 @@ it; the CUDA library never does, and this package imports nothing from it.
 Every function works in float64 on inputs upcast from the stored bf16/fp32
 bytes, and never rounds an intermediate.
 """
-from . import philox, views, drafter, sampler  # noqa: F401
+from . import philox, views, drafter, sampler, verify  # noqa: F401
 from .views import OracleState, state_init, view_update, full_summary, state_bytes_per_request  # noqa: F401
 from .drafter import OracleWeights, draft_base_logits  # noqa: F401
 from .sampler import sample_block, gumbel  # noqa: F401
+from .verify import verify_block  # noqa: F401
