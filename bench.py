@@ -249,6 +249,41 @@ def prefill_leg(wl, rows, hbm, dist, reps=5):
                     "tensor-issue bound on the legacy path, not HBM"}
 
 
+def verify_leg(wl, hbm, dist, reps=20):
+    """lsp_verify of one round's blocks against (synthetic) target logits [C][B+1][V]:
+    device time and HBM fraction at T = 1 (residual / bonus draws) and T = 0 (greedy)."""
+    s, lsp = wl.s, wl.lsp
+    zt, _ = synth.make_verify_logits(s, seed=wl.seed_base + 9500)
+    zt = zt.cuda()
+    acc = torch.zeros(s.C, dtype=torch.int32, device="cuda")
+    tok = torch.zeros(s.C, dtype=torch.int32, device="cuda")
+    st = wl.new_state()
+    out = {"C": s.C, "B": s.B, "V": s.V}
+    for name, T in (("T1", 1.0), ("T0", 0.0)):
+        sp = lsp.make_sample_params(T, seed=synth.RNG_SEED, rnd=1)
+        for _ in range(3):
+            lsp.lsp_verify(st, zt, wl.logits, wl.toks, sp, acc, tok)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        dist.barrier()
+        e0.record()
+        for _ in range(reps):
+            lsp.lsp_verify(st, zt, wl.logits, wl.toks, sp, acc, tok)
+        e1.record()
+        torch.cuda.synchronize()
+        us = dist.max(e0.elapsed_time(e1) * 1e3 / reps)
+        # every row read once for its statistics, plus the emitting rows re-read by the draw
+        rows = s.C * (2 * s.B + 3) if T > 0 else s.C * (s.B + 1)
+        nbytes = rows * s.V * 4
+        out[name] = {"us": us, "bytes": nbytes, "achieved_gbs": nbytes / us * 1e-3,
+                     "frac_hbm": nbytes / us * 1e-3 / hbm}
+    assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+    lsp.lsp_state_destroy(st)
+    out["note"] = ("inputs %.0f MB > L2 (no flush needed); T = 1 reads target and draft rows, "
+                   "T = 0 the target rows only" % (s.C * (2 * s.B + 1) * s.V * 4 / 1e6))
+    return out
+
+
 # ------------------------------------------------------------------ workload
 class Workload:
     def __init__(self, s, lsp, seed_base):
@@ -562,6 +597,10 @@ def run_ours(args, dist):
     if prefixes and not args.no_sweep and s.dtype == "bf16":
         prefill = prefill_leg(wl, max(prefixes), hbm, dist)
 
+    verify = None
+    if not args.no_sweep:
+        verify = verify_leg(wl, hbm, dist)
+
     cpu = None
     if want_cpu:
         leg = oracle_leg(wl, kept, args.cpu_budget)
@@ -578,7 +617,8 @@ def run_ours(args, dist):
            "e2e": {"value": dist.world * s.C * s.B / (e2e_ms * 1e-3), "unit": UNIT,
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
            "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
-           "clocks": clocks, "sweep": sweep, "prefill": prefill, "cpu_baseline": cpu}
+           "clocks": clocks, "sweep": sweep, "prefill": prefill, "verify": verify,
+           "cpu_baseline": cpu}
     if dist.rank == 0:
         print(json.dumps(out), flush=True)
     lsp.lsp_state_destroy(st)

@@ -256,6 +256,30 @@ int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, cons
  * LSP_ERR_UNSUPPORTED: use lsp_view_update).  Other requests are untouched. */
 int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream);
 
+/* Target-side verification of the drafted blocks (Sec. 2.1, Eq. acceptance,
+ * Eq. residual): for each request the candidates y_1..y_B are tested in order,
+ * y_i accepted with probability min(1, p_i(y_i) / q_i(y_i)); at the first
+ * rejected position i a correction token is drawn from [p_i - q_i]_+; if all B
+ * are accepted a bonus token is drawn from p_{B+1}.  p_i = softmax(target
+ * logits_i / T), q_i = softmax(draft logits_i / T); T = 0 is greedy (accept
+ * y_i iff y_i = argmax p_i, emit argmax p_{r+1}; ties to the lowest index).
+ *   target_logits: device float [C][B+1][V] (position B: p(. | s, y_1..y_B));
+ *   draft_logits: device float [C][B][V] (lsp_draft's out_logits);
+ *   draft_tokens: device int32 [C][B] (lsp_draft's out_tokens);
+ *   sp: the round's sampling parameters (the ones lsp_draft used);
+ *   accepted_len: device int32 [C] = r in [0, B]; next_token: device int32 [C].
+ *   16-byte aligned logits.  The round then advances each request by r + 1
+ *   tokens (the next round's accepted_len is r + 1 and its committed token is
+ *   next_token).
+ * Randomness: Philox4x32-10 with key `seed`; acceptance uniform of position i =
+ * word 0 of counter (0, 2^30 + i, b, round), u = ((x >> 9) + 1/2) 2^-23,
+ * accepted iff u q_i(y_i) < p_i(y_i); the draw at position i is Gumbel-max with
+ * the words of counters (v >> 2, 2^31 + i, b, round).  Drafted tokens outside
+ * [0, V) set LSP_DEV_BAD_TOKEN.  Asynchronous on `stream`. */
+int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_logits,
+               const int32_t* draft_tokens, const lsp_sample_params* sp, int32_t* accepted_len,
+               int32_t* next_token, lsp_stream_t stream);
+
 /* Dense projection Y = X W^T with the drafter's tensor-core GEMM (the kernel
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].

@@ -44,19 +44,6 @@ constexpr int kSampWarps = kSampThreads / 32;
 constexpr int kMaxC = 64;
 constexpr int kMaxPartialsPerLane = 16;    // sampler grids of up to 512 CTAs
 
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
-  const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u;
-  const uint32_t W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    const uint32_t hi0 = __umulhi(M0, c.x), lo0 = M0 * c.x;
-    const uint32_t hi1 = __umulhi(M1, c.z), lo1 = M1 * c.z;
-    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
-    k.x += W0;
-    k.y += W1;
-  }
-  return c;
-}
 
 // g = -log(-log u): the inner log keeps full relative accuracy (u can be within
 // 2^-24 of 1, where -log u is tiny); the outer log only needs absolute accuracy.

@@ -71,6 +71,12 @@ struct lsp_state {
   float* part_val = nullptr;
   int* part_idx = nullptr;
   float* prefill_ws = nullptr;       // prefill segment partials (bf16, d = 128 configs)
+  float* ver_sa = nullptr;           // verification row partials and draw partials
+  float* ver_sb = nullptr;
+  int* ver_si = nullptr;
+  float* ver_pv = nullptr;
+  int* ver_pi = nullptr;
+  unsigned* ver_ctr = nullptr;
   unsigned long long* sample_sync = nullptr;
   size_t sample_sync_bytes = 0;
   int nblk = 0;
@@ -228,6 +234,13 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   const size_t w_sync = off; off = align256(off + sample_sync_bytes(c.B));
   const bool prefill_ok = c.dtype == LSP_DTYPE_BF16 && c.d == 128;
   const size_t w_pf = off; off = align256(off + (prefill_ok ? prefill_ws_floats(c.L, c.nq) * sizeof(float) : 0));
+  const size_t ver_rows = (size_t)c.C * (2 * c.B + 1) * verify_max_stat_chunks(c.V);
+  const size_t w_vsa = off; off = align256(off + ver_rows * sizeof(float));
+  const size_t w_vsb = off; off = align256(off + ver_rows * sizeof(float));
+  const size_t w_vsi = off; off = align256(off + ver_rows * sizeof(int));
+  const size_t w_vpv = off; off = align256(off + (size_t)c.C * kVerMaxDrawChunks * sizeof(float));
+  const size_t w_vpi = off; off = align256(off + (size_t)c.C * kVerMaxDrawChunks * sizeof(int));
+  const size_t w_vc = off; off = align256(off + (size_t)c.C * sizeof(unsigned));
   if (cudaMalloc(&st->ws, off) != cudaSuccess) { free_state(st); return LSP_ERR_NOMEM; }
   char* w = static_cast<char*>(st->ws);
   st->x = reinterpret_cast<float*>(w + w_x);
@@ -243,6 +256,12 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   st->part_idx = reinterpret_cast<int*>(w + w_pi);
   st->sample_sync = reinterpret_cast<unsigned long long*>(w + w_sync);
   st->prefill_ws = prefill_ok ? reinterpret_cast<float*>(w + w_pf) : nullptr;
+  st->ver_sa = reinterpret_cast<float*>(w + w_vsa);
+  st->ver_sb = reinterpret_cast<float*>(w + w_vsb);
+  st->ver_si = reinterpret_cast<int*>(w + w_vsi);
+  st->ver_pv = reinterpret_cast<float*>(w + w_vpv);
+  st->ver_pi = reinterpret_cast<int*>(w + w_vpi);
+  st->ver_ctr = reinterpret_cast<unsigned*>(w + w_vc);
   st->sample_sync_bytes = sample_sync_bytes(c.B);
   if (cudaMemset(st->ws, 0, off) != cudaSuccess || cudaMemset(st->base, 0, o_done + l.done) != cudaSuccess) {
     free_state(st);
@@ -315,6 +334,25 @@ int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t st
   p.ws = st->prefill_ws;
   p.b = b; p.L = c.L; p.nq = c.nq; p.nkv = c.nkv; p.d = c.d; p.W = c.W; p.R = c.R; p.H = c.H;
   return launch_prefill(p, c.dtype, S(stream));
+}
+
+int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_logits,
+               const int32_t* draft_tokens, const lsp_sample_params* sp, int32_t* accepted_len,
+               int32_t* next_token, lsp_stream_t stream) {
+  if (!st || !target_logits || !draft_logits || !draft_tokens || !sp || !accepted_len || !next_token)
+    return LSP_ERR_ARG;
+  if (!(sp->temperature >= 0.f) || !std::isfinite(sp->temperature)) return LSP_ERR_ARG;
+  if (((uintptr_t)target_logits | (uintptr_t)draft_logits) & 15) return LSP_ERR_ARG;
+  const lsp_config& c = st->cfg;
+  VerifyParams p;
+  p.zt = target_logits; p.zq = draft_logits; p.y = draft_tokens;
+  p.accepted = accepted_len; p.next_token = next_token;
+  p.st_a = st->ver_sa; p.st_b = st->ver_sb; p.st_i = st->ver_si; p.nst = 1;
+  p.part_val = st->ver_pv; p.part_idx = st->ver_pi;
+  p.ctr = st->ver_ctr; p.err = st->err;
+  p.C = c.C; p.B = c.B; p.V = c.V;
+  p.temperature = sp->temperature; p.round = sp->round; p.seed = sp->seed;
+  return launch_verify(p, st->num_sms, S(stream));
 }
 
 static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {

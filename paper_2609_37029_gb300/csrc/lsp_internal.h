@@ -175,6 +175,32 @@ constexpr int kPrefillMaxSeg = 64;   // prefix segments (CTAs per tapped layer x
 size_t prefill_ws_floats(int L, int nq);
 int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s);
 
+// ------------------------------------------------------------------ verification
+struct VerifyParams {
+  const float* zt;          // target logits [C][B+1][V]
+  const float* zq;          // draft logits [C][B][V]
+  const int32_t* y;         // drafted tokens [C][B]
+  int32_t* accepted;        // [C]
+  int32_t* next_token;      // [C]
+  float* st_a;              // chunk partials [C][2B+1][nst]: max of z log2(e) / T (T > 0), max of z (T = 0)
+  float* st_b;              //   sum of 2^(x - max) (T > 0)
+  int* st_i;                //   argmax index (T = 0)
+  int nst;                  // chunks per row (set by launch_verify)
+  float* part_val;          // draw partials [C][<= kVerMaxDrawChunks]
+  int* part_idx;
+  unsigned* ctr;            // [C] self-resetting counters (zero between calls)
+  unsigned* err;
+  int C, B, V;
+  float temperature;
+  uint32_t round;
+  uint64_t seed;
+};
+constexpr int kVerMaxStatChunks = 32;
+constexpr int kVerMaxDrawChunks = 128;
+constexpr int kVerMaxB = 512;
+int verify_max_stat_chunks(int V);
+int launch_verify(const VerifyParams& p, int num_sms, cudaStream_t s);
+
 // ------------------------------------------------------------------ sampler
 struct SampleParams {
   const float* src;       // [C][B][V] base logits

@@ -78,6 +78,8 @@ _f = {
     "lsp_view_update": _sig("lsp_view_update", c_int, c_void_p, POINTER(lsp_target_feats), c_void_p,
                             c_void_p),
     "lsp_prefill": _sig("lsp_prefill", c_int, c_void_p, c_int, POINTER(lsp_target_feats), c_void_p),
+    "lsp_verify": _sig("lsp_verify", c_int, c_void_p, c_void_p, c_void_p, c_void_p,
+                       POINTER(lsp_sample_params), c_void_p, c_void_p, c_void_p),
     "lsp_draft": _sig("lsp_draft", c_int, c_void_p, c_void_p, POINTER(lsp_weights),
                       POINTER(lsp_sample_params), c_void_p, c_void_p, c_void_p),
     "lsp_sample": _sig("lsp_sample", c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -188,6 +190,13 @@ def lsp_prefill(st, b, k, v, h, rows=None, stream=None) -> None:
     """k, v: [L][t][nkv][d], h: [L][t][H] of request b's whole prefix."""
     f = lsp_target_feats(_ptr(k), _ptr(v), _ptr(h), int(rows if rows is not None else k.shape[1]))
     _check(_f["lsp_prefill"](st, int(b), ctypes.byref(f), _stream(stream)), "lsp_prefill")
+
+
+def lsp_verify(st, target_logits, draft_logits, draft_tokens, sp: lsp_sample_params, accepted_len,
+               next_token, stream=None) -> None:
+    _check(_f["lsp_verify"](st, _ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens),
+                            ctypes.byref(sp), _ptr(accepted_len), _ptr(next_token), _stream(stream)),
+           "lsp_verify")
 
 
 def lsp_draft(st, block_tokens, weights: lsp_weights, sp: lsp_sample_params, out_tokens,

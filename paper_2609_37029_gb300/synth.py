@@ -202,3 +202,20 @@ def make_block_tokens(shape: LspShape, seed: int, device="cpu"):
     bt = torch.full((shape.C, shape.B), -1, dtype=torch.int32)
     bt[:, 0] = torch.randint(0, shape.V, (shape.C,), generator=g, dtype=torch.int32)
     return bt.to(device)
+
+
+def make_verify_logits(shape: LspShape, seed: int, std: float = 2.0, agree=(0.9, 0.999)):
+    """Target and draft logits of one verification call, fp32.
+
+    zt [C][B+1][V] ~ N(0, std^2); the draft row i of request b is
+    a_b zt[b, i] + sqrt(1 - a_b^2) N(0, std^2) with a_b ~ U[agree]: requests range
+    from a drafter that mostly agrees with the target to one that often does not,
+    so the accepted lengths spread over [0, B].
+    """
+    g = _gen(seed, "cpu")
+    C, B, V = shape.C, shape.B, shape.V
+    zt = torch.randn((C, B + 1, V), generator=g, dtype=torch.float32) * std
+    a = agree[0] + (agree[1] - agree[0]) * torch.rand((C, 1, 1), generator=g, dtype=torch.float64)
+    noise = torch.randn((C, B, V), generator=g, dtype=torch.float32) * std
+    zq = (a * zt[:, :B].double() + torch.sqrt(1 - a * a) * noise.double()).float()
+    return zt.contiguous(), zq.contiguous()
