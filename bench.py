@@ -284,6 +284,32 @@ def verify_leg(wl, hbm, dist, reps=20):
     return out
 
 
+def variants_leg(s, lsp, seed_base, dist, steps=100, prefix=4096):
+    """Round time of the paper's B = 7 and of the three ablation variants (Sec. 3.4) on
+    the same kernels: drafted tokens/s and the per-request interface bytes."""
+    out = {}
+    for name, kw in (("B7", {"B": 7}), ("no_window", {"W": 0}), ("no_summary", {"R": 0}),
+                     ("no_boundary", {"no_boundary": True})):
+        sv = s.with_(**kw)
+        wl = Workload(sv, lsp, seed_base + 300)
+        st = wl.new_state()
+        wl.fold(st, 0, prefix)
+        for _ in range(2):
+            wl.round(st)
+        g = wl.capture(st)
+        ms, _ = time_graph(g, steps, 10, dist)
+        ms = dist.max(ms)
+        assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+        out[name] = {"us_per_round": ms * 1e3, "drafted_tokens_per_s": dist.world * sv.C * sv.B / (ms * 1e-3),
+                     "state_bytes": lsp.lsp_state_bytes(wl.cfg), "launches": lsp.lsp_round_launches(st)}
+        del g
+        lsp.lsp_state_destroy(st)
+        del wl
+        torch.cuda.empty_cache()
+    out["note"] = "prefix %d rows folded; same weights recipe; W = 0 / R = 0 / no boundary remove one context source" % prefix
+    return out
+
+
 # ------------------------------------------------------------------ workload
 class Workload:
     def __init__(self, s, lsp, seed_base):
@@ -294,7 +320,7 @@ class Workload:
         self.cfg = lsp.make_config(s)
         rows = s.B + 1
         self.k, self.v, self.h = synth.make_features(s, rows, seed=seed_base + 5000, device="cuda")
-        self.acc = synth.make_accepted(s, seed=seed_base + 5001, device="cuda")
+        self.acc = synth.make_accepted(s, seed=seed_base + 5001, device="cuda", hi=min(s.delta_max, s.B + 1))
         self.bt = synth.make_block_tokens(s, seed=seed_base + 5002, device="cuda")
         self.toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
         self.logits = torch.empty(s.C, s.B, s.V, device="cuda")
@@ -601,6 +627,10 @@ def run_ours(args, dist):
     if not args.no_sweep:
         verify = verify_leg(wl, hbm, dist)
 
+    variants = None
+    if not args.no_sweep and s.dtype == "bf16":
+        variants = variants_leg(s, lsp, wl.seed_base, dist)
+
     cpu = None
     if want_cpu:
         leg = oracle_leg(wl, kept, args.cpu_budget)
@@ -618,7 +648,7 @@ def run_ours(args, dist):
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
            "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
            "clocks": clocks, "sweep": sweep, "prefill": prefill, "verify": verify,
-           "cpu_baseline": cpu}
+           "variants": variants, "cpu_baseline": cpu}
     if dist.rank == 0:
         print(json.dumps(out), flush=True)
     lsp.lsp_state_destroy(st)

@@ -60,6 +60,13 @@ extern "C" {
 #define LSP_DTYPE_BF16 0
 #define LSP_DTYPE_F32 1
 
+/* lsp_config.flags.  LSP_NO_BOUNDARY: the "w/o boundary state" variant of the
+ * ablation (Sec. 3.4, Fig. 5): the state keeps no boundary hidden state, the
+ * boundary fusion is not run and the input slots are E[u_i] + P_i alone.  The
+ * other two variants are shapes: w/o global summary is R = 0, w/o recent KV
+ * window is W = 0. */
+#define LSP_NO_BOUNDARY 1u
+
 typedef void* lsp_stream_t;       /* cudaStream_t */
 typedef struct lsp_state lsp_state; /* opaque, library-owned */
 
@@ -78,8 +85,10 @@ typedef struct lsp_state lsp_state; /* opaque, library-owned */
  *       from (Sec. 2.3 pairs draft layer j with tapped layer l(j)); a value < 0
  *       selects floor(j * L / D)
  *   rope_theta  rotary base of the drafter's block queries/keys; rms_eps RMSNorm eps
+ *   flags  0 or LSP_NO_BOUNDARY
  * Supported: dtype BF16 with d == 128, B <= 16, nq % nkv == 0, nq/nkv <= 8;
- * dtype F32 with d <= 128 even; H, nq*d, nkv*d, F multiples of 64; C*B <= 512.
+ * dtype F32 with d <= 128 even; H, nq*d, nkv*d, F multiples of 64; C*B <= 512;
+ * W >= 0 and R >= 0 (0 removes the window / the summary from the context).
  */
 typedef struct lsp_config {
   int C, B, L, D, H, nq, nkv, d, F, V, W, R, rc;
@@ -87,6 +96,7 @@ typedef struct lsp_config {
   int layer_map[LSP_MAX_DRAFT_LAYERS];
   float rope_theta;
   float rms_eps;
+  unsigned flags;
 } lsp_config;
 
 /*
@@ -95,7 +105,8 @@ typedef struct lsp_config {
  *   k[b][l][j][0..nkv)[0..d)   key rows as cached by the target (rotary applied)
  *   v[b][l][j][0..nkv)[0..d)   value rows
  *   h[b][l][j][0..H)           hidden state at that row (only row accepted_len-1 is read)
- * All three are device pointers of dtype with row capacity `rows` per (b, l).
+ * All three are device pointers of dtype with row capacity `rows` per (b, l);
+ * h may be null (and is not read) with LSP_NO_BOUNDARY.
  */
 typedef struct lsp_target_feats {
   const void* k;
@@ -125,7 +136,8 @@ typedef struct lsp_weights {
   const void* embed;       /* [V][H] target token embedding */
   const void* final_norm;  /* [H] target final RMSNorm weight */
   const void* lm_head;     /* [V][H] target vocabulary head */
-  const void* fuse;        /* [H][L*H] boundary fusion: c_t = fuse . [h^l1;...;h^lL] (Sec. 2.2) */
+  const void* fuse;        /* [H][L*H] boundary fusion: c_t = fuse . [h^l1;...;h^lL] (Sec. 2.2);
+                              may be null with LSP_NO_BOUNDARY */
   const void* pos;         /* [B][H] within-block positional encodings (Sec. 2.3) */
   const void* mask_emb;    /* [H] mask-token embedding of slots 1..B-1 */
   const void* Ec;          /* [V][rc] correction embedding E_c (Eq. markov) */
@@ -252,7 +264,7 @@ int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, cons
  * Equivalent to folding the t rows into an empty request with
  * lsp_view_update, but split over the whole GPU (segments of the prefix
  * merged in order with Eq. summary-update; deterministic).  Needs an
- * initialised state (G); bf16 storage with d = 128, R <= 16, nq/nkv <= 8 (else
+ * initialised state (G); bf16 storage with d = 128, 0 <= R <= 16, nq/nkv <= 8 (else
  * LSP_ERR_UNSUPPORTED: use lsp_view_update).  Other requests are untouched. */
 int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream);
 
@@ -304,7 +316,8 @@ int lsp_philox_words(uint64_t seed, uint32_t round, uint32_t b, uint32_t i,
  * stage boundaries on the call's stream: stage k runs between events[k] and
  * events[k+1].  Stages of one round, in order (lsp_stage_count / lsp_stage_name):
  *   0 view_update, 1 fuse, 2 combine, then per draft layer j: qkv, attention,
- *   o_proj, post_norm, gate_up, down, next_norm, then lm_head and sampler.
+ *   o_proj, post_norm, gate_up, down, next_norm, then lm_head and sampler
+ *   (with LSP_NO_BOUNDARY the fuse stage is empty).
  * n_events must be 0 (off) or lsp_stage_count(st) + 1.  Event records are
  * capturable, so a captured round carries them as graph nodes. */
 int lsp_stage_count(lsp_state* st);

@@ -121,11 +121,17 @@ def draft_layer(cfg, lw, x, pos, kw, vw, Gl, ml):
 
 
 def draft_hidden(cfg, st, w: OracleWeights, block_tokens, b):
-    """Final hidden rows [B][H] of request b (before the frozen final norm)."""
-    c = boundary_state(cfg, w, st.hb[b])
+    """Final hidden rows [B][H] of request b (before the frozen final norm).
+
+    The "w/o boundary state" variant of the ablation (Sec. 3.4, Fig. 5) drops
+    c_t from the input slots: x_i = E[u_i] + P_i.  (W = 0 and R = 0 are the
+    variants without the recent window and without the global summary.)
+    """
     emb = np.stack([w.embed_row(int(u)) if int(u) >= 0 else w.mask_emb
                     for u in block_tokens[b]])
-    x = emb + w.pos + c[None, :]
+    x = emb + w.pos
+    if not getattr(cfg, "no_boundary", False):
+        x = x + boundary_state(cfg, w, st.hb[b])[None, :]
     pos = int(st.t[b]) + np.arange(cfg.B)
     for j in range(cfg.D):
         l = cfg.layer_map[j]

@@ -120,10 +120,11 @@ def state_bytes_per_request(cfg, elem_bytes=2):
 
     window K and V in the storage dtype: L * W * 2 * nkv * d elements;
     summary (m, eta) in fp32: L * nq * R * (d + 1) floats ("one value vector and
-    one log-normalizer per query", App. A.2); boundary h: L * H elements.
+    one log-normalizer per query", App. A.2); boundary h: L * H elements
+    (none in the ablation variant without the boundary state, Sec. 3.4).
     Independent of t (Sec. 2.4, "Fixed-cost complexity").
     """
     win = cfg.L * cfg.W * 2 * cfg.nkv * cfg.d * elem_bytes
     summ = cfg.L * cfg.nq * cfg.R * (cfg.d + 1) * 4
-    bnd = cfg.L * cfg.H * elem_bytes
+    bnd = 0 if getattr(cfg, "no_boundary", False) else cfg.L * cfg.H * elem_bytes
     return win + summ + bnd

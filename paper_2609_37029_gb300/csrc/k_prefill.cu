@@ -266,10 +266,12 @@ __global__ void __launch_bounds__(256) prefill_merge_kernel(const PrefillParams 
     *reinterpret_cast<uint4*>(wv + slot) = *reinterpret_cast<const uint4*>(vin + (size_t)q * rstride + c);
   }
   if (g == 0) {
-    const T* hin = static_cast<const T*>(p.hid) + ((size_t)l * p.rows + (p.rows - 1)) * p.H;
-    T* hout = static_cast<T*>(p.h) + ((size_t)b * p.L + l) * p.H;
-    for (int i = threadIdx.x * vec; i < p.H; i += blockDim.x * vec)
-      *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
+    if (p.h) {   // no boundary state is kept with LSP_NO_BOUNDARY
+      const T* hin = static_cast<const T*>(p.hid) + ((size_t)l * p.rows + (p.rows - 1)) * p.H;
+      T* hout = static_cast<T*>(p.h) + ((size_t)b * p.L + l) * p.H;
+      for (int i = threadIdx.x * vec; i < p.H; i += blockDim.x * vec)
+        *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
+    }
     if (l == 0 && threadIdx.x == 0) p.t[b] = p.rows;
   }
 }
@@ -278,7 +280,7 @@ size_t prefill_ws_floats(int L, int nq) { return (size_t)kPrefillMaxSeg * L * nq
 
 int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s) {
   const int rep = p.nq / p.nkv;
-  if (dtype != LSP_DTYPE_BF16 || p.d != kPfD || p.R > 16 || p.R < 1 || rep > 8 || p.rows < 1 || !p.ws)
+  if (dtype != LSP_DTYPE_BF16 || p.d != kPfD || p.R > 16 || p.R < 0 || rep > 8 || p.rows < 1 || !p.ws)
     return LSP_ERR_UNSUPPORTED;
   if (p.H % 8) return LSP_ERR_SHAPE;
   // segments of a multiple of 64 rows, at most kPrefillMaxSeg of them
@@ -294,8 +296,9 @@ int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s) {
       return LSP_ERR_CUDA;
     attr = smem;
   }
-  if (launch_pdl(prefill_partial_kernel, dim3(nseg, p.L * p.nkv), dim3(rep * 32), smem, s, p, rep,
-                 seg_rows) != cudaSuccess ||
+  // R = 0 (no summary): only the window, boundary and t are written
+  if ((p.R > 0 && launch_pdl(prefill_partial_kernel, dim3(nseg, p.L * p.nkv), dim3(rep * 32), smem, s, p,
+                             rep, seg_rows) != cudaSuccess) ||
       launch_pdl(prefill_merge_kernel<bf16>, dim3(p.L * p.nq + p.L * p.nkv), dim3(256), 0, s, p, nseg) !=
           cudaSuccess)
     return LSP_ERR_CUDA;

@@ -102,7 +102,8 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
                         : static_cast<const T*>(p.mask_emb);
   const T* pos = static_cast<const T*>(p.pos) + (size_t)i * p.H;
   const size_t cstride = (size_t)p.C * p.H;
-  const float* c = p.c + (size_t)b * p.H;
+  // c_t split partials (absent with LSP_NO_BOUNDARY: c == nullptr, c_splits == 0)
+  const float* c = p.c ? p.c + (size_t)b * p.H : nullptr;
   const int h4 = p.H / 4;
   float4 xv[kMaxVec];
   float ss = 0.f;
@@ -110,7 +111,7 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   for (int k = 0; k < kMaxVec; ++k) {
     const int j = threadIdx.x + k * kRowThreads;
     if (j < h4) {
-      float4 cv = ld4(c, j);
+      float4 cv = c ? ld4(c, j) : make_float4(0.f, 0.f, 0.f, 0.f);
       for (int s0 = 1; s0 < p.c_splits; s0 += 4) {
         float4 t[4];
 #pragma unroll

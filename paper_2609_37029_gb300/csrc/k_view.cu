@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kViewThreads)
   }
 
   // ---- boundary: hidden state of the last new row, this CTA's 1/nkv share
-  {
+  if (p.h) {   // no boundary state is kept with LSP_NO_BOUNDARY
     const T* hin = static_cast<const T*>(p.h_new) +
                    ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
     T* hout = static_cast<T*>(p.h) + (size_t)(b * p.L + l) * p.H;

@@ -33,7 +33,7 @@ Layout interface_layout(const lsp_config& c) {
   l.win = (size_t)c.C * c.L * c.nkv * c.W * c.d * es;
   l.m = (size_t)c.C * c.L * c.nq * c.R * c.d * sizeof(float);
   l.eta = (size_t)c.C * c.L * c.nq * c.R * sizeof(float);
-  l.h = (size_t)c.C * c.L * c.H * es;
+  l.h = (c.flags & LSP_NO_BOUNDARY) ? 0 : (size_t)c.C * c.L * c.H * es;
   l.t = (size_t)c.C * sizeof(int64_t);
   l.G = (size_t)c.L * c.nq * c.R * c.d * es;
   l.err = sizeof(unsigned);
@@ -122,6 +122,7 @@ int lsp_config_check(const lsp_config* c) {
       c->d < 2 || c->F < 1 || c->V < 1 || c->W < 0 || c->R < 0 || c->rc < 1)
     return LSP_ERR_SHAPE;
   if (c->dtype != LSP_DTYPE_BF16 && c->dtype != LSP_DTYPE_F32) return LSP_ERR_ARG;
+  if (c->flags & ~LSP_NO_BOUNDARY) return LSP_ERR_ARG;
   if (c->D > LSP_MAX_DRAFT_LAYERS || c->nq % c->nkv) return LSP_ERR_SHAPE;
   if (c->C * c->B > 512 || c->C > 64) return LSP_ERR_SHAPE;
   if (c->H % 128 || (c->nq * c->d) % 128 || (c->nkv * c->d) % 128 || c->F % 64) return LSP_ERR_SHAPE;
@@ -200,7 +201,7 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   st->win_k = b + o_wk; st->win_v = b + o_wv;
   st->m = reinterpret_cast<float*>(b + o_m);
   st->eta = reinterpret_cast<float*>(b + o_eta);
-  st->h = b + o_h;
+  st->h = l.h ? b + o_h : nullptr;
   st->t = reinterpret_cast<int64_t*>(b + o_t);
   st->G = b + o_G;
   st->err = reinterpret_cast<unsigned*>(b + o_err);
@@ -288,15 +289,14 @@ __global__ void state_reset_kernel(float* eta, size_t n_eta, int64_t* t, int C, 
 }
 
 int lsp_state_init(lsp_state* st, const void* G, lsp_stream_t stream) {
-  if (!st || !G) return LSP_ERR_ARG;
+  if (!st) return LSP_ERR_ARG;
   const lsp_config& c = st->cfg;
   const Layout l = interface_layout(c);
+  if (!G && l.G) return LSP_ERR_ARG;          // G is empty (may be null) when R = 0
   cudaStream_t s = S(stream);
-  if (cudaMemsetAsync(st->win_k, 0, l.win, s) != cudaSuccess ||
-      cudaMemsetAsync(st->win_v, 0, l.win, s) != cudaSuccess ||
-      cudaMemsetAsync(st->m, 0, l.m, s) != cudaSuccess ||
-      cudaMemsetAsync(st->h, 0, l.h, s) != cudaSuccess ||
-      cudaMemcpyAsync(st->G, G, l.G, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+  auto zero = [&](void* p, size_t n) { return n == 0 || cudaMemsetAsync(p, 0, n, s) == cudaSuccess; };
+  if (!zero(st->win_k, l.win) || !zero(st->win_v, l.win) || !zero(st->m, l.m) || !zero(st->h, l.h) ||
+      (l.G && cudaMemcpyAsync(st->G, G, l.G, cudaMemcpyDeviceToDevice, s) != cudaSuccess))
     return LSP_ERR_CUDA;
   const size_t n_eta = l.eta / sizeof(float);
   const size_t n = std::max(n_eta, (size_t)c.C);
@@ -309,7 +309,8 @@ int lsp_state_init(lsp_state* st, const void* G, lsp_stream_t stream) {
 
 int lsp_view_update(lsp_state* st, const lsp_target_feats* f, const int32_t* acc,
                     lsp_stream_t stream) {
-  if (!st || !f || !acc || !f->k || !f->v || !f->h || f->rows < 1) return LSP_ERR_ARG;
+  if (!st || !f || !acc || !f->k || !f->v || f->rows < 1) return LSP_ERR_ARG;
+  if (!f->h && st->h) return LSP_ERR_ARG;
   if (!st->initialized) return LSP_ERR_STATE;
   const lsp_config& c = st->cfg;
   ViewParams p;
@@ -324,7 +325,8 @@ int lsp_view_update(lsp_state* st, const lsp_target_feats* f, const int32_t* acc
 }
 
 int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream) {
-  if (!st || !f || !f->k || !f->v || !f->h || f->rows < 1) return LSP_ERR_ARG;
+  if (!st || !f || !f->k || !f->v || f->rows < 1) return LSP_ERR_ARG;
+  if (!f->h && st->h) return LSP_ERR_ARG;
   if (!st->initialized) return LSP_ERR_STATE;
   const lsp_config& c = st->cfg;
   if (b < 0 || b >= c.C) return LSP_ERR_ARG;
@@ -368,7 +370,8 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
       return LSP_ERR_SHAPE;
     return r;
   };
-  {
+  if (st->h) {
+    if (!w->fuse) return LSP_ERR_ARG;
     const void* W[1] = {w->fuse};
     const int rows[1] = {c.H};
     if ((rc = plan(&st->fuse, st->h, c.C, c.L * c.H, W, rows, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
@@ -441,13 +444,13 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   }
   const int M = c.C * c.B;
   int ev = 2;   // stage boundaries after view_update's [0, 1]
-  // boundary state c_t = W_fuse [h^l1; ...; h^lL]
-  if ((rc = gemm_launch(&st->fuse, s)) != LSP_OK) return rc;
+  // boundary state c_t = W_fuse [h^l1; ...; h^lL] (absent with LSP_NO_BOUNDARY)
+  if (st->h && (rc = gemm_launch(&st->fuse, s)) != LSP_OK) return rc;
   mark(st, ev++, s);
   // input slots + first input norm + rotary table
   CombineParams cp;
   cp.tokens = block_tokens; cp.embed = w->embed; cp.pos = w->pos; cp.mask_emb = w->mask_emb;
-  cp.c = st->part; cp.c_splits = st->fuse.p.splits; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
+  cp.c = st->h ? st->part : nullptr; cp.c_splits = st->h ? st->fuse.p.splits : 0; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
   cp.t = st->t; cp.err = st->err; cp.C = c.C; cp.B = c.B; cp.H = c.H; cp.V = c.V; cp.d = c.d;
   cp.eps = c.rms_eps; cp.theta = (double)c.rope_theta;
   if ((rc = launch_combine(cp, c.dtype, s)) != LSP_OK) return rc;
@@ -543,7 +546,8 @@ int lsp_round_launches(lsp_state* st) {
   p.C = c.C; p.B = c.B; p.V = c.V; p.rc = c.rc; p.num_sms = st->num_sms; p.sync = st->sample_sync;
   // view update, fuse, combine; per layer q/k/v GEMM + finalize, attention, o, norm, gate/up, down,
   // norm; LM head; the sampler
-  return 3 + 8 * c.D + 1 + sample_launches(p, c.dtype);
+  const int fuse = (c.flags & LSP_NO_BOUNDARY) ? 0 : 1;
+  return 2 + fuse + 8 * c.D + 1 + sample_launches(p, c.dtype);
 }
 
 const char* lsp_stage_name(lsp_state* st, int k) {
@@ -594,6 +598,7 @@ static int copy_interface(lsp_state* st, void* host, size_t bytes, bool to_host,
   void* dev[6] = {st->win_k, st->win_v, st->m, st->eta, st->h, st->t};
   const size_t sz[6] = {l.win, l.win, l.m, l.eta, l.h, l.t};
   for (int i = 0; i < 6; ++i) {
+    if (sz[i] == 0) continue;
     cudaError_t e = to_host ? cudaMemcpyAsync(hp, dev[i], sz[i], cudaMemcpyDeviceToHost, s)
                             : cudaMemcpyAsync(dev[i], hp, sz[i], cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return LSP_ERR_CUDA;

@@ -20,6 +20,7 @@ LSP_MAX_DRAFT_LAYERS = 16
 LSP_OK, LSP_ERR_ARG, LSP_ERR_SHAPE, LSP_ERR_CUDA = 0, -1, -2, -3
 LSP_ERR_TIMEOUT, LSP_ERR_STATE, LSP_ERR_NOMEM, LSP_ERR_UNSUPPORTED = -4, -5, -6, -7
 LSP_DEV_TIMEOUT, LSP_DEV_BAD_TOKEN, LSP_DEV_BAD_DELTA = 1, 2, 4
+LSP_NO_BOUNDARY = 1
 LSP_DTYPE_BF16, LSP_DTYPE_F32 = 0, 1
 
 if not os.path.exists(LIB_PATH):
@@ -30,7 +31,8 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 class lsp_config(Structure):
     _fields_ = [(n, c_int) for n in "C B L D H nq nkv d F V W R rc dtype".split()] + [
-        ("layer_map", c_int * LSP_MAX_DRAFT_LAYERS), ("rope_theta", c_float), ("rms_eps", c_float)]
+        ("layer_map", c_int * LSP_MAX_DRAFT_LAYERS), ("rope_theta", c_float), ("rms_eps", c_float),
+        ("flags", c_uint32)]
 
 
 class lsp_target_feats(Structure):
@@ -135,6 +137,7 @@ def make_config(shape) -> lsp_config:
         c.layer_map[j] = int(lm[j]) if j < len(lm) else -1
     c.rope_theta = float(shape.rope_theta)
     c.rms_eps = float(shape.rms_eps)
+    c.flags = LSP_NO_BOUNDARY if getattr(shape, "no_boundary", False) else 0
     return c
 
 

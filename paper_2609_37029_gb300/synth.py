@@ -53,6 +53,7 @@ class LspShape:
     outlier_mult: float = 1.0
     delta_max: int = 16             # accepted_len ~ U[1, delta_max]
     layer_map: tuple = ()           # draft layer j -> tapped index (default floor(j*L/D))
+    no_boundary: bool = False       # ablation: no boundary state / fusion (W = 0, R = 0: the others)
 
     def __post_init__(self):
         if not self.layer_map:

@@ -46,7 +46,7 @@ def export_state(lsp, st, s):
              ("win_v", s.C * s.L * s.nkv * s.W * s.d * es, dt, (s.C, s.L, s.nkv, s.W, s.d)),
              ("m", s.C * s.L * s.nq * s.R * s.d * 4, torch.float32, (s.C, s.L, s.nq, s.R, s.d)),
              ("eta", s.C * s.L * s.nq * s.R * 4, torch.float32, (s.C, s.L, s.nq, s.R)),
-             ("h", s.C * s.L * s.H * es, dt, (s.C, s.L, s.H)),
+             ("h", 0 if s.no_boundary else s.C * s.L * s.H * es, dt, (s.C, s.L, 0 if s.no_boundary else s.H)),
              ("t", s.C * 8, torch.int64, (s.C,))]
     out, off = {}, 0
     for name, nb, t, shp in sizes:
@@ -73,7 +73,8 @@ def check_view_state(lsp, st, ost, s, atol_m=1e-4):
     assert list(ex["t"].numpy()) == list(ost.t)
     np.testing.assert_allclose(ex["m"].double().numpy(), ost.m, rtol=0, atol=atol_m)
     np.testing.assert_allclose(ex["eta"].double().numpy(), ost.eta, rtol=0, atol=atol_m * 10)
-    assert np.array_equal(f64(ex["h"]), ost.hb)
+    if not s.no_boundary:                                      # the variant keeps no boundary
+        assert np.array_equal(f64(ex["h"]), ost.hb)
     wk, wv = f64(ex["win_k"]), f64(ex["win_v"])
     for b in range(s.C):
         t = int(ost.t[b])

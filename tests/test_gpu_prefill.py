@@ -52,6 +52,33 @@ def test_prefill_matches_oracle(lsp, t):
         lsp.lsp_state_destroy(st)
 
 
+@pytest.mark.parametrize("variant", [{"R": 0}, {"W": 0}, {"no_boundary": True}])
+def test_prefill_ablation_variants(lsp, variant):
+    """Without the summary (R = 0) only the window, boundary and t are written; without the
+    window (W = 0) only the summary; without the boundary no hidden state is read (h = None)."""
+    s = PF.with_(**variant)
+    st = lsp.lsp_state_create(lsp.make_config(s))
+    try:
+        w = synth.make_weights(s, seed=3)
+        lsp.lsp_state_init(st, w["G"].cuda() if w["G"].numel() else None)
+        ost = oracle.state_init(s)
+        Gn = f64(w["G"])
+        t = 777
+        k, v, h = synth.make_features(s, t, seed=55)
+        hb = None if s.no_boundary else h[1].contiguous().cuda()
+        lsp.lsp_prefill(st, 1, k[1].contiguous().cuda(), v[1].contiguous().cuda(), hb)
+        fresh = oracle.state_init(s.with_(C=1))
+        oracle.view_update(s.with_(C=1), fresh, Gn, f64(k[1:2]), f64(v[1:2]), f64(h[1:2]),
+                           np.array([t], dtype=np.int32))
+        ost.eta[1], ost.m[1], ost.hb[1], ost.t[1] = fresh.eta[0], fresh.m[0], fresh.hb[0], fresh.t[0]
+        ost.win_k[1], ost.win_v[1] = fresh.win_k[0], fresh.win_v[0]
+        torch.cuda.synchronize()
+        check_view_state(lsp, st, ost, s)
+        assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+    finally:
+        lsp.lsp_state_destroy(st)
+
+
 def test_prefill_replaces_state_and_rounds_continue(lsp):
     """A prefill overwrites a request that already holds rows; later view updates fold on top."""
     s = PF

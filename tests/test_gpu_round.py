@@ -91,6 +91,19 @@ def test_round_matches_oracle(lsp, name):
     _run_round(lsp, s, s.prefix)
 
 
+@pytest.mark.parametrize("variant", [
+    {"B": 7},                                   # the paper's block size
+    {"W": 0},                                   # ablation: w/o recent KV window (Sec. 3.4)
+    {"R": 0},                                   # ablation: w/o global summary
+    {"no_boundary": True},                      # ablation: w/o boundary state
+    {"B": 7, "W": 0, "R": 0, "no_boundary": True, "temperature": 1.0},
+])
+def test_round_variants_match_oracle(lsp, variant):
+    """The paper's B = 7 and the three ablation variants through the same kernels."""
+    s = synth.SMALL.with_(**variant)
+    _run_round(lsp, s, 3000)
+
+
 def test_round_sampled_and_short_prefix(lsp):
     """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
     s = synth.SMALL.with_(temperature=1.0)

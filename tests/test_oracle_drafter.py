@@ -186,20 +186,35 @@ def test_draft_matches_explicit_loop_brute_force():
         np.testing.assert_allclose(z0[b], ref, rtol=1e-11, atol=1e-12)
 
 
-def test_draft_matches_torch_composition():
-    """The same pass assembled from torch fp64 library calls (linear, rms_norm, SDPA, silu)."""
-    cfg = MICRO.with_(H=32, d=16, nq=4, nkv=2, F=48, V=64, W=8, R=4, D=3, L=2)
+TORCH_CFG = MICRO.with_(H=32, d=16, nq=4, nkv=2, F=48, V=64, W=8, R=4, D=3, L=2)
+
+
+@pytest.mark.parametrize("variant", [
+    {},                                  # the full drafter
+    {"B": 7},                            # the paper's block size (7 drafts per round)
+    {"W": 0},                            # ablation: w/o recent KV window (Sec. 3.4)
+    {"R": 0},                            # ablation: w/o global summary
+    {"no_boundary": True},               # ablation: w/o boundary state
+    {"W": 0, "R": 0, "no_boundary": True},
+])
+def test_draft_matches_torch_composition(variant):
+    """The same pass assembled from torch fp64 library calls (linear, rms_norm, SDPA, silu),
+    for the full drafter and each variant of the ablation (a removed source is simply absent
+    from the concatenated keys and values; without the boundary state the input slots carry
+    no c_t)."""
+    cfg = TORCH_CFG.with_(**variant)
     st, G = _state(cfg, 13, 7)
     w = _np_weights(cfg, seed=8)
     w["G"] = G
-    toks = np.array([[1, -1, -1, -1], [63, -1, -1, 2]])
+    toks = np.array([[1] + [-1] * (cfg.B - 2) + [2], [63] + [-1] * (cfg.B - 1)])
     z0 = oracle.draft_base_logits(cfg, st, oracle.OracleWeights(w), toks)
     T = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
     rep = cfg.nq // cfg.nkv
     for b in range(cfg.C):
-        c = Fn.linear(T(st.hb[b]).reshape(-1), T(w["fuse"]))
         emb = torch.stack([T(w["embed"][t]) if t >= 0 else T(w["mask_emb"]) for t in toks[b]])
-        x = emb + T(w["pos"]) + c
+        x = emb + T(w["pos"])
+        if not cfg.no_boundary:
+            x = x + Fn.linear(T(st.hb[b]).reshape(-1), T(w["fuse"]))
         pos = torch.arange(cfg.B, dtype=torch.float64) + float(st.t[b])
         inv = cfg.rope_theta ** (-torch.arange(0, cfg.d, 2, dtype=torch.float64) / cfg.d)
         ang = pos[:, None] * inv[None, :]
@@ -223,6 +238,30 @@ def test_draft_matches_torch_composition():
             x = x + Fn.linear(Fn.silu(Fn.linear(xn, lw["w_gate"])) * Fn.linear(xn, lw["w_up"]), lw["w_down"])
         ref = Fn.linear(Fn.rms_norm(x, (cfg.H,), T(w["final_norm"]), cfg.rms_eps), T(w["lm_head"]))
         np.testing.assert_allclose(z0[b], ref.numpy(), rtol=1e-11, atol=1e-12)
+
+
+def test_without_boundary_equals_a_zero_fusion_matrix():
+    """The no-boundary variant is the full drafter with W_fuse = 0, whatever h holds."""
+    cfg = TORCH_CFG
+    st, G = _state(cfg, 11, 12)
+    w = _np_weights(cfg, seed=13)
+    w["G"] = G
+    toks = np.array([[5, -1, -1, -1], [9, -1, 4, -1]])
+    z_nb = oracle.draft_base_logits(cfg.with_(no_boundary=True), st, oracle.OracleWeights(w), toks)
+    w0 = dict(w, fuse=np.zeros_like(w["fuse"]))
+    z_0 = oracle.draft_base_logits(cfg, st, oracle.OracleWeights(w0), toks)
+    np.testing.assert_allclose(z_nb, z_0, rtol=1e-13, atol=1e-13)
+    # and the boundary does matter for the full drafter
+    assert np.abs(oracle.draft_base_logits(cfg, st, oracle.OracleWeights(w), toks) - z_0).max() > 1e-3
+
+
+def test_state_bytes_of_the_ablation_variants():
+    """Each removed source removes exactly its bytes from the per-request interface."""
+    s = synth.Q8B
+    full = oracle.state_bytes_per_request(s)
+    assert full - oracle.state_bytes_per_request(s.with_(W=0)) == s.L * s.W * 2 * s.nkv * s.d * 2
+    assert full - oracle.state_bytes_per_request(s.with_(R=0)) == s.L * s.nq * s.R * (s.d + 1) * 4
+    assert full - oracle.state_bytes_per_request(s.with_(no_boundary=True)) == s.L * s.H * 2
 
 
 def test_layer_pairing_reads_its_tapped_layer():
