@@ -296,10 +296,14 @@ int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_log
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].
  *   M <= 512; K * element size a multiple of 16 bytes.
- *   splits: split-K factor (1..16, at most the number of K blocks); with
- *   splits > 1 the kernel writes fp32 partial sums to `workspace` (device, at
+ *   splits: split-K factor (1..16, at most the number of K blocks).  The
+ *   kernel writes fp32 partial sums to `workspace` (device, at
  *   least lsp_linear_workspace_bytes(M, N, splits) bytes) and a second kernel
- *   sums them in split order into Y. */
+ *   sums them in split order into Y.  With the environment variable
+ *   LSP_GEMM_CLUSTER=1 and splits 2, 4 or 8 instead, the split CTAs of each
+ *   128-row weight tile form a thread-block cluster that sums its partials in
+ *   distributed shared memory, in split order, and writes Y (workspace unused;
+ *   the drafter's projections then reduce the same way). */
 size_t lsp_linear_workspace_bytes(int M, int N, int splits);
 int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype,
                int splits, void* workspace, size_t workspace_bytes, lsp_stream_t stream);

@@ -165,6 +165,88 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
   if (issuer) bulk_wait_read<0>();                            // staging smem is released at exit
 }
 
+// Split-K reduction inside the cluster (all threads of the CTA call it the
+// same number of times; one weight tile per CTA).  Pass by pass over
+// cr_tok-token chunks of the accumulator: the epilogue warps dump their TMEM
+// rows into this CTA's idle stage ring as [token][128 rows] fp32; after a
+// cluster barrier, the CTA of cluster rank k sums the k-th token slice of the
+// chunk over the split CTAs in split order (deterministic) through
+// distributed shared memory and writes the final output; a second barrier
+// frees the dumps for the next pass.
+template <typename T>
+__device__ __forceinline__ void epilogue_cluster(const GemmParams& p, uint8_t* smem, uint32_t tmem_base,
+                                                 int tile, bool have_acc) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int s = p.splits;
+  const uint32_t rank = cluster_ctarank();
+  float* dump = reinterpret_cast<float*>(smem);
+  const uint32_t dump_u32 = smem_u32(dump);
+  const bool swiglu = p.mode == EPI_SWIGLU;
+  const bool f32out = p.mode == EPI_F32 || p.mode == EPI_PARTIAL;
+  const int q = warp & 3, r = q * 32 + lane;                  // TMEM lane = weight row
+  const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
+  const int groups = swiglu ? 16 : 32;                        // float4 row groups per token
+  for (int p0 = 0; p0 < p.m_pad; p0 += p.cr_tok) {
+    const int np = min(p.cr_tok, p.m_pad - p0);
+    if (warp >= 2 && have_acc) {
+      for (int c0 = 0; c0 < np; c0 += 16) {
+        float v[16];
+        tmem_ld16(lane_base + (uint32_t)(p0 + c0), v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) dump[(c0 + j) * kTileRows + r] = v[j];
+      }
+    }
+    cluster_sync_all();
+    const int tl = (np + s - 1) / s;
+    const int t0 = (int)rank * tl, t1 = min(t0 + tl, np);
+    for (int g = threadIdx.x; g < (t1 - t0) * groups; g += blockDim.x) {
+      const int t = t0 + g / groups, r4 = (g % groups) * 4;
+      const int m = p0 + t;
+      if (m >= p.M) continue;
+      // every peer's value in flight at once, then the sum in split order
+      float4 xa[kMaxClusterSplits], xu[kMaxClusterSplits];
+      const uint32_t off = dump_u32 + (uint32_t)((t * kTileRows + r4) * 4);
+#pragma unroll
+      for (int k = 0; k < kMaxClusterSplits; ++k)
+        if (k < s) {
+          xa[k] = ld_dsmem_f4(off, (uint32_t)k);
+          if (swiglu) xu[k] = ld_dsmem_f4(off + 64 * 4, (uint32_t)k);
+        }
+      float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
+#pragma unroll
+      for (int k = 0; k < kMaxClusterSplits; ++k)
+        if (k < s) {
+          a.x += xa[k].x; a.y += xa[k].y; a.z += xa[k].z; a.w += xa[k].w;
+          if (swiglu) { u.x += xu[k].x; u.y += xu[k].y; u.z += xu[k].z; u.w += xu[k].w; }
+        }
+      const float av[4] = {a.x, a.y, a.z, a.w}, uv[4] = {u.x, u.y, u.z, u.w};
+      if (swiglu) {
+        T* Y = static_cast<T*>(p.Y) + (size_t)m * p.ldy;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int f = tile * 64 + r4 + e;
+          if (f < p.N) Y[f] = from_f<T>(av[e] / (1.0f + expf(-av[e])) * uv[e]);
+        }
+      } else if (f32out) {
+        float* Y = static_cast<float*>(p.Y) + (size_t)m * p.ldy;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int n = tile * kTileRows + r4 + e;
+          if (n < p.N) Y[n] = av[e];
+        }
+      } else {
+        T* Y = static_cast<T*>(p.Y) + (size_t)m * p.ldy;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int n = tile * kTileRows + r4 + e;
+          if (n < p.N) Y[n] = from_f<T>(av[e]);
+        }
+      }
+    }
+    cluster_sync_all();
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap ta0, const __grid_constant__ CUtensorMap ta1,
@@ -319,7 +401,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_fence_after();
     named_bar(1, 128);
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
-    if (*s_abort == 0 && p.tma_out) {
+    if (p.creduce) {
+      // reduced across the cluster below, by the whole CTA
+    } else if (*s_abort == 0 && p.tma_out) {
       epilogue_tma<T>(p, &to, smem, lane_base, ntl, tile0, split, r);
     } else if (*s_abort == 0) {
       for (int w = 0; w < ntl; ++w)
@@ -338,6 +422,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // A wait gave up: let every TMA copy this CTA issued land before exit.
     for (int i = (issued > S ? issued - S : 0); i < issued; ++i)
       mbar_wait(full_bar(i % S), (uint32_t)(i / S) & 1u, p.err);
+  }
+  if (p.creduce) {
+    // the stage ring is idle: every load landed before the last MMA was issued
+    // (or, after an abort, in the drain above); the dumps reuse it
+    __syncthreads();
+    tc_fence_after();
+    epilogue_cluster<T>(p, smem, tmem_base, tile0, *s_abort == 0);
+    tc_fence_before();
   }
   if (warp == 1) {
     tc_fence_after();
@@ -453,22 +545,24 @@ static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
 
 // Split-K factor from a cost model in units of one k-block of one of two
 // co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
-// fixed per-CTA cost) + the consumer's re-read of the fp32 split partials
-// from L2 (partial_cost per split).  With a small token tile a lone CTA on an
-// SM streams a k-block in ~0.63 of that time; with a wide one (>= 128 tokens)
-// a lone CTA is no faster: its single MMA issuer keeps the tensor pipe only
+// fixed per-CTA cost) + the cost of combining the splits (fixed_cost +
+// per_split_cost per split: the consumer's re-read of fp32 partials from L2,
+// or the in-cluster reduction).  With a small token tile a lone CTA on an SM
+// streams a k-block in ~0.63 of that time; with a wide one (>= 128 tokens) a
+// lone CTA is no faster: its single MMA issuer keeps the tensor pipe only
 // partly busy, and a second CTA on the SM hides that.
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok,
-                     bool wide) {
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
+                     int max_splits, bool two_ok, bool wide) {
   double best = 1e30;
   int splits = 1;
-  for (int s = 1; s <= std::min(16, kblocks); ++s) {
+  for (int s = 1; s <= std::min(max_splits, kblocks); ++s) {
+    if (max_splits == kMaxClusterSplits && s > 1 && (s & (s - 1))) continue;   // cluster sizes 2, 4, 8
     const long long ctas = (long long)n_ctas * s;
     const bool two = two_ok && ctas * 4 >= (long long)num_sms * 5;
     const long long slots = two ? 2LL * num_sms : num_sms;
     const long long waves = (ctas + slots - 1) / slots;
     const double per = (double)((kblocks + s - 1) / s) * (two || wide ? 1.0 : 0.63) + 2.0;
-    const double cost = (double)waves * per + (s > 1 ? partial_cost * s : 0.0);
+    const double cost = (double)waves * per + (s > 1 ? fixed_cost + per_split_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
   return splits;
@@ -478,6 +572,21 @@ int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, 
 // model's k-block units (~1.56 us).
 double gemm_partial_cost(int M, int N) { return (double)M * N * 4.0 / 5e12 / 1.56e-6; }
 
+// Split-K reduced inside thread-block clusters, opt-in (LSP_GEMM_CLUSTER=1).
+// Measured at the Qwen3-8B drafting round it is slower than partial sums
+// through L2 (o_proj 28 vs 19.5 us per launch, round 1.41 vs 1.27 ms): the
+// distributed-shared-memory reduction runs at the tail, after the slowest
+// split, and its ~112 KB of peer reads per CTA are slow; so partials stay the
+// default and the clustered path is kept for other shapes and for testing.
+bool gemm_cluster_enabled() {
+  const char* v = std::getenv("LSP_GEMM_CLUSTER");
+  return v && v[0] == '1';
+}
+
+// Model cost of one in-cluster reduction, k-block units: two cluster barriers
+// per pass and the distributed-shared-memory reads of the peers' dumps.
+constexpr double kClusterReduceCost = 1.5;
+
 void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt) {
   int bn, ntt;
   token_tiling(M, &bn, &ntt);
@@ -486,11 +595,16 @@ void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, in
   if (*wt <= 0) *wt = 1;
   const int kblocks = gemm_kblocks(K, dtype);
   const int n_ctas = (n_tiles + *wt - 1) / *wt;
-  if (*splits <= 0)
-    *splits = mode == EPI_PARTIAL
-                  ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows),
-                                     two_per_sm_fits(*wt, m_pad), m_pad >= 128)
-                  : 1;
+  const bool two = two_per_sm_fits(*wt, m_pad), wide = m_pad >= 128;
+  if (*splits <= 0) {
+    if (gemm_cluster_enabled() && *wt == 1)
+      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, 0.0, kClusterReduceCost, kMaxClusterSplits, two, wide);
+    else if (mode == EPI_PARTIAL)
+      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows), 0.0, 16,
+                                 two, wide);
+    else
+      *splits = 1;
+  }
   *splits = std::max(1, std::min(*splits, kblocks));
 }
 
@@ -541,8 +655,15 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   // (distance 1: 318 -> 281 us at the LM-head shape; longer distances were slower)
   p.pd = 1;
   if (std::getenv("LSP_GEMM_PD")) p.pd = std::max(0, tuning("LSP_GEMM_PD"));
-  if (splits > 1 && mode != EPI_PARTIAL) return LSP_ERR_SHAPE;
   p.splits = splits;
+  // split-K: reduced in a cluster of the tile's split CTAs when possible
+  // (power-of-two clusters: a cluster of 6 measured 23 co-resident clusters, not 48)
+  p.creduce = (splits == 2 || splits == 4 || splits == 8) && wt == 1 && gemm_cluster_enabled() ? 1 : 0;
+  if (splits > 1 && mode != EPI_PARTIAL && !p.creduce) return LSP_ERR_SHAPE;
+  p.out_splits = p.creduce ? 1 : splits;
+  // tokens per reduction pass: the stage ring holds a [tokens][128] fp32 dump
+  p.cr_tok = std::min(p.m_pad, (int)((size_t)p.stages * stage_bytes / (kTileRows * 4) / 16 * 16));
+  if (p.creduce && p.cr_tok < 16) return LSP_ERR_SHAPE;
   p.Y = Y;
   p.ldy = ldy;
   p.err = err;
@@ -559,11 +680,12 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   {
     const bool f32 = mode == EPI_F32 || mode == EPI_PARTIAL || dtype == LSP_DTYPE_F32;
     const int cols = mode == EPI_SWIGLU ? 64 : kTileRows;
-    p.tma_out = make_out_map(&op->out, f32, Y, p.N, M, splits, ldy, cols, p.out_tok) == LSP_OK &&
+    p.tma_out = make_out_map(&op->out, f32, Y, p.N, M, p.out_splits, ldy, cols, p.out_tok) == LSP_OK &&
                 std::getenv("LSP_GEMM_SCALAR_EPI") == nullptr;
     if (!p.tma_out) op->out = op->b;       // unused placeholder
   }
   op->grid = dim3((unsigned)n_ctas, (unsigned)splits, 1);
+  op->cluster = p.creduce ? splits : 1;
   op->smem = (size_t)p.stages * stage_bytes + 1024 + 256;
   return LSP_OK;
 }
@@ -574,8 +696,28 @@ static int launch_t(const GemmOp* op, cudaStream_t s) {
   std::call_once(once, [] {
     cudaFuncSetAttribute(gemm_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
   });
-  const cudaError_t e = launch_pdl(gemm_kernel<T>, op->grid, dim3(kGemmThreads), op->smem, s,
-                                   op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
+  if (op->cluster <= 1) {
+    const cudaError_t e = launch_pdl(gemm_kernel<T>, op->grid, dim3(kGemmThreads), op->smem, s,
+                                     op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
+    return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
+  }
+  // the split CTAs of a weight tile form one cluster (grid.y == cluster size)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = op->grid;
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = op->smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = (unsigned)op->cluster;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_kernel<T>, op->a[0], op->a[1], op->a[2], op->b,
+                                           op->out, op->p);
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 

@@ -366,7 +366,7 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
                   int nseg, int mode, void* Y, int ldy) {
     const int r = gemm_plan(op, dt, X, Mx, K, W, rows, nseg, mode, Y, ldy, st->err, st->num_sms, 0, 0);
     if (r == LSP_OK && mode == EPI_PARTIAL &&
-        (size_t)op->p.splits * Mx * op->p.N * sizeof(float) > st->part_bytes)
+        (size_t)op->p.out_splits * Mx * op->p.N * sizeof(float) > st->part_bytes)
       return LSP_ERR_SHAPE;
     return r;
   };
@@ -450,7 +450,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   // input slots + first input norm + rotary table
   CombineParams cp;
   cp.tokens = block_tokens; cp.embed = w->embed; cp.pos = w->pos; cp.mask_emb = w->mask_emb;
-  cp.c = st->h ? st->part : nullptr; cp.c_splits = st->h ? st->fuse.p.splits : 0; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
+  cp.c = st->h ? st->part : nullptr; cp.c_splits = st->h ? st->fuse.p.out_splits : 0; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
   cp.t = st->t; cp.err = st->err; cp.C = c.C; cp.B = c.B; cp.H = c.H; cp.V = c.V; cp.d = c.d;
   cp.eps = c.rms_eps; cp.theta = (double)c.rope_theta;
   if ((rc = launch_combine(cp, c.dtype, s)) != LSP_OK) return rc;
@@ -459,7 +459,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     const lsp_layer_weights& lw = w->layer[j];
     if ((rc = gemm_launch(&st->qkv_op[j], s)) != LSP_OK) return rc;
     QkvParams qp;
-    qp.part = st->part; qp.splits = st->qkv_op[j].p.splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
+    qp.part = st->part; qp.splits = st->qkv_op[j].p.out_splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
     qp.rope = st->rope; qp.out = st->qkv; qp.M = M; qp.B = c.B; qp.nq = c.nq; qp.nkv = c.nkv; qp.d = c.d;
     qp.eps = c.rms_eps;
     if ((rc = launch_qkv_finalize(qp, c.dtype, s)) != LSP_OK) return rc;
@@ -473,7 +473,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->o_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
-    if ((rc = launch_resid_norm(st->x, st->part, st->o_op[j].p.splits, lw.post_norm, st->xn, M, c.H,
+    if ((rc = launch_resid_norm(st->x, st->part, st->o_op[j].p.out_splits, lw.post_norm, st->xn, M, c.H,
                                 c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
@@ -482,7 +482,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     if ((rc = gemm_launch(&st->down_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
     const void* next_norm = j + 1 < c.D ? w->layer[j + 1].in_norm : w->final_norm;
-    if ((rc = launch_resid_norm(st->x, st->part, st->down_op[j].p.splits, next_norm, st->xn, M, c.H,
+    if ((rc = launch_resid_norm(st->x, st->part, st->down_op[j].p.out_splits, next_norm, st->xn, M, c.H,
                                 c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
@@ -523,11 +523,13 @@ int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int 
   GemmOp op;
   const void* Ws[1] = {W};
   float* part = static_cast<float*>(workspace);
-  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, splits > 1 ? EPI_PARTIAL : EPI_F32,
-                     splits > 1 ? part : Y, N, nullptr, sms, splits, 0);
+  // splits <= 8: reduced inside a cluster straight into Y; else partials + a sum kernel
+  const bool in_cluster = splits == 1 || ((splits == 2 || splits == 4 || splits == 8) && gemm_cluster_enabled());
+  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, in_cluster ? EPI_F32 : EPI_PARTIAL,
+                     in_cluster ? Y : part, N, nullptr, sms, splits, 0);
   if (rc != LSP_OK) return rc;
   if (op.p.splits != splits) return LSP_ERR_SHAPE;
-  if ((rc = gemm_launch(&op, S(stream))) != LSP_OK || splits == 1) return rc;
+  if ((rc = gemm_launch(&op, S(stream))) != LSP_OK || in_cluster) return rc;
   return launch_sum_partials(part, splits, (size_t)M * N, Y, S(stream));
 }
 

@@ -51,6 +51,10 @@ struct GemmParams {
   int bn, n_tok_tiles, m_pad, stages, tmem_cols, pd;
   int tma_out;          // 1: the epilogue stages tiles in shared memory and TMA-stores them
   int out_tok;          // tokens per staged output chunk (16 or 32)
+  int creduce;          // 1: the `splits` CTAs of a tile form a cluster and reduce split-K in
+                        //    distributed shared memory; the output is final (one slice)
+  int cr_tok;           // tokens per cluster-reduction pass (the idle stage ring holds them)
+  int out_splits;       // slices of the output the consumer sums (splits, or 1 when reduced)
   void* Y;
   int ldy;
   unsigned* err;
@@ -63,13 +67,18 @@ struct GemmOp {
   GemmParams p;
   int dtype;
   dim3 grid;
+  int cluster;          // CTAs per cluster along the split axis (1: no cluster)
   size_t smem;
 };
 
 // Plan Y = X W^T where W is the row-concatenation of `nseg` weight segments
 // (each [seg_rows[i]][K]); for EPI_SWIGLU, segment 0 = gate and 1 = up, both
-// [N][K].  EPI_PARTIAL writes `splits` partial sums [splits][M][ldy]; other
-// modes need splits == 1.  splits <= 0 / wt <= 0 choose for `num_sms`.
+// [N][K].  With splits > 1 the split-K partial sums are reduced inside a
+// thread-block cluster (splits <= kMaxClusterSplits) and every mode writes its
+// final output (EPI_PARTIAL then writes one fp32 slice: p.out_splits == 1);
+// otherwise EPI_PARTIAL writes `splits` partial sums [splits][M][ldy] for the
+// consumer to add and other modes need splits == 1.  splits <= 0 / wt <= 0
+// choose for `num_sms`.
 int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
               const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
               int num_sms, int splits, int wt);
@@ -77,8 +86,10 @@ int gemm_launch(const GemmOp* op, cudaStream_t s);
 // The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 = choose).
 void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double partial_cost, bool two_ok,
-                     bool wide);
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
+                     int max_splits, bool two_ok, bool wide);
+constexpr int kMaxClusterSplits = 8;    // portable cluster size
+bool gemm_cluster_enabled();
 double gemm_partial_cost(int M, int N);
 int gemm_kblocks(int K, int dtype);
 // Deterministic sum of `splits` fp32 partials [splits][n] into y[n].

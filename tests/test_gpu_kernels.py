@@ -47,13 +47,26 @@ LINEAR_CASES = [
     (256, 640, 1000, "bf16", 4),
     (300, 200, 136, "bf16", 1),
     (512, 256, 512, "bf16", 2),
+    (256, 512, 4096, "bf16", 8),     # cluster of 8, two reduction passes
+    (16, 384, 20480, "bf16", 8),     # the boundary-fusion shape (M = C)
+    (200, 256, 2048, "bf16", 4),     # ragged token count, uneven token slices
+    (96, 256, 1024, "bf16", 5),      # a split count no cluster takes: partials + sum kernel
+    (256, 256, 1024, "bf16", 12),    # beyond a cluster: partials through L2 + sum kernel
     (8, 128, 256, "f32", 1),
     (64, 384, 260, "f32", 3),
+    (64, 384, 520, "f32", 2),
 ]
 
 
+@pytest.mark.parametrize("cluster", [False, True])
 @pytest.mark.parametrize("M,N,K,dt,splits", LINEAR_CASES)
-def test_linear_matches_fp64_matmul(lsp, M, N, K, dt, splits):
+def test_linear_matches_fp64_matmul(lsp, M, N, K, dt, splits, cluster, monkeypatch):
+    """Split-K through fp32 partials and a sum kernel, or (LSP_GEMM_CLUSTER=1, splits 2/4/8)
+    reduced inside a thread-block cluster through distributed shared memory."""
+    if cluster:
+        if splits not in (2, 4, 8):
+            pytest.skip("no cluster for this split count")
+        monkeypatch.setenv("LSP_GEMM_CLUSTER", "1")
     g = torch.Generator().manual_seed(M * 7 + N + K)
     tdt = torch.bfloat16 if dt == "bf16" else torch.float32
     X = torch.randn(M, K, generator=g).to(tdt)
@@ -62,11 +75,15 @@ def test_linear_matches_fp64_matmul(lsp, M, N, K, dt, splits):
     nbytes = lsp.lsp_linear_workspace_bytes(M, N, splits)
     ws = torch.zeros(max(nbytes, 4), dtype=torch.uint8, device="cuda")
     code = lsp.LSP_DTYPE_BF16 if dt == "bf16" else lsp.LSP_DTYPE_F32
+    prev = None
     for _ in range(2):              # second call reuses the workspace (counters reset)
         lsp.lsp_linear(X.cuda(), W.cuda(), Y, M, N, K, code, splits, ws, nbytes)
         torch.cuda.synchronize()
         ref = f64(X) @ f64(W).T
         got = f64(Y)
+        if prev is not None:        # split-K sums in a fixed order: bit-identical reruns
+            assert np.array_equal(got, prev)
+        prev = got.copy()
         scale = np.abs(ref).max()
         # bf16 operands are exact; tf32 rounds operands to 10 mantissa bits
         tol = 1e-5 if dt == "bf16" else 4e-3

@@ -104,6 +104,14 @@ def test_round_variants_match_oracle(lsp, variant):
     _run_round(lsp, s, 3000)
 
 
+def test_round_with_cluster_split_k(lsp, monkeypatch):
+    """The projections' split-K reduced inside thread-block clusters (opt-in) gives the
+    same round within the same tolerance."""
+    monkeypatch.setenv("LSP_GEMM_CLUSTER", "1")
+    s = synth.SMALL.with_(temperature=1.0)
+    _run_round(lsp, s, 2500)
+
+
 def test_round_sampled_and_short_prefix(lsp):
     """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
     s = synth.SMALL.with_(temperature=1.0)
