@@ -14,8 +14,11 @@
 // read of the window and summary); warps are (query head x key split); each
 // warp runs an online softmax over 16-key chunks with mma.sync m16n8k16
 // (bf16 in, fp32 accumulate), and the key splits merge through shared memory.
-// attn_simple_kernel (fp32 storage): plain FMA version, one CTA per
-// (request, query head), for the fp32 reference shape.
+// attn_simple_kernel (fp32 storage): FMA version, one CTA per (request, query
+// head), for the fp32 reference shape: window and summary rows are staged in
+// shared memory 64 at a time (float4 loads, several in flight per thread), a
+// warp scores each staged key against all block queries (lanes split over
+// queries and head dims), one softmax, then P V over the re-staged values.
 #include <type_traits>
 
 #include "common.cuh"
@@ -269,10 +272,38 @@ __global__ void __launch_bounds__(512)
 }
 
 // ------------------------------------------------------------ fp32 reference shape
+constexpr int kSimpleChunk = 64;    // window / summary rows staged per round trip
+
+// Rows [j0, j0 + nr) of the context list "count window rows, then summary rows"
+// into shared memory as [nr][d] floats: float4 loads (d % 4 == 0), four in
+// flight per thread before their stores.
+__device__ __forceinline__ void stage_rows(float* dst, const float* win, const float* summ, int count,
+                                           int j0, int nr, int d) {
+  const int d4 = d / 4, n4 = nr * d4;
+  for (int base = threadIdx.x; base < n4; base += 4 * blockDim.x) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = base + u * blockDim.x;
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (idx < n4) {
+        const int r = j0 + idx / d4, c4 = idx % d4;
+        const float* src = r < count ? win + (size_t)r * d : summ + (size_t)(r - count) * d;
+        v[u] = reinterpret_cast<const float4*>(src)[c4];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < n4) reinterpret_cast<float4*>(dst)[idx] = v[u];
+    }
+  }
+}
+
 template <typename T>
-__global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
   extern __shared__ float ssm[];
-  const int d = p.d, B = p.B, half = d / 2;
+  const int d = p.d, B = p.B;
   const int rep = p.nq / p.nkv;
   const int b = blockIdx.x / p.nq, h = blockIdx.x % p.nq, g = h / rep;
   const long long t = p.t[b];
@@ -283,7 +314,6 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
   float* sv = sk + B * d;
   float* ss = sv + B * d;                 // [B][ctx]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
-  (void)lane;
   griddep_launch();
   griddep_wait();
   const T* qkv = static_cast<const T*>(p.qkv);
@@ -302,21 +332,36 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
   const T* Gh = static_cast<const T*>(p.G) + ((size_t)p.layer * p.nq + h) * p.R * d;
   const float* Mh = p.m + (((size_t)(b * p.L + p.layer) * p.nq + h) * p.R) * d;
   const float scale = rsqrtf((float)d);
-  for (int idx = tid; idx < B * ctx; idx += blockDim.x) {
-    const int i = idx / ctx, j = idx % ctx;
-    float acc = 0.f;
-    if (j < B) {
-      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * sk[j * d + e];
-    } else if (j < B + count) {
-      const T* kr = wk + (size_t)(j - B) * d;
-      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * to_f(kr[e]);
-    } else {
-      const T* kr = Gh + (size_t)(j - B - count) * d;
-      for (int e = 0; e < d; ++e) acc += sq[i * d + e] * to_f(kr[e]);
+  float* sc = ss + ((size_t)B * ctx + 3) / 4 * 4;   // [kSimpleChunk][d] staged rows (16-B aligned)
+  const int nctx = count + p.R;           // window rows, then summary rows
+  // Lanes split into groups of `lpq` per block query (lpq = the largest power
+  // of two with lpq * B <= 32, queries in passes of 32 / lpq); lane c of a
+  // group covers dims c, c + lpq, ... so a score needs log2(lpq) shuffles.
+  int lpq = 1;
+  while (lpq * 2 * B <= 32) lpq *= 2;
+  const int qpp = 32 / lpq, qi = lane / lpq, c = lane % lpq;
+  auto score = [&](const float* krow, int j) {   // j: context index of the key
+    for (int i0 = 0; i0 < B; i0 += qpp) {
+      const int i = i0 + qi;
+      float part = 0.f;
+      if (i < B)
+        for (int e = c; e < d; e += lpq) part = fmaf(sq[i * d + e], krow[e], part);
+      for (int o = lpq / 2; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+      if (i < B && c == 0) ss[i * ctx + j] = part * scale;
     }
-    ss[idx] = acc * scale;
+  };
+  // ---- scores: block keys from shared memory, then the window and summary
+  // keys staged kSimpleChunk rows at a time (one coalesced round trip each)
+  for (int j = warp; j < B; j += nw) score(sk + j * d, j);
+  for (int j0 = 0; j0 < nctx; j0 += kSimpleChunk) {
+    const int nr = min(kSimpleChunk, nctx - j0);
+    __syncthreads();
+    stage_rows(sc, wk, Gh, count, j0, nr, d);
+    __syncthreads();
+    for (int r = warp; r < nr; r += nw) score(sc + r * d, B + j0 + r);
   }
   __syncthreads();
+  // ---- one softmax per query over the B + count + R scores
   for (int i = warp; i < B; i += nw) {
     float mx = -INFINITY;
     for (int j = lane; j < ctx; j += 32) mx = fmaxf(mx, ss[i * ctx + j]);
@@ -331,18 +376,33 @@ __global__ void __launch_bounds__(128) attn_simple_kernel(const AttnParams p) {
     for (int j = lane; j < ctx; j += 32) ss[i * ctx + j] /= sum;
   }
   __syncthreads();
+  // ---- P V, accumulated in place of the (no longer needed) queries: block
+  // values first, then the window and summary values staged like the keys
+  float* acc = sq;
+  for (int idx = tid; idx < B * d; idx += blockDim.x) {
+    const int i = idx / d, e = idx % d;
+    float a = 0.f;
+    for (int j = 0; j < B; ++j) a = fmaf(ss[i * ctx + j], sv[j * d + e], a);
+    acc[idx] = a;
+  }
+  for (int j0 = 0; j0 < nctx; j0 += kSimpleChunk) {
+    const int nr = min(kSimpleChunk, nctx - j0);
+    __syncthreads();
+    stage_rows(sc, wv, Mh, count, j0, nr, d);
+    __syncthreads();
+    for (int idx = tid; idx < B * d; idx += blockDim.x) {
+      const int i = idx / d, e = idx % d;
+      const float* pr = ss + (size_t)i * ctx + B + j0;
+      float a = acc[idx];
+      for (int r = 0; r < nr; ++r) a = fmaf(pr[r], sc[r * d + e], a);
+      acc[idx] = a;
+    }
+  }
+  __syncthreads();
   T* out = static_cast<T*>(p.out);
   for (int idx = tid; idx < B * d; idx += blockDim.x) {
     const int i = idx / d, e = idx % d;
-    float acc = 0.f;
-    for (int j = 0; j < ctx; ++j) {
-      float v;
-      if (j < B) v = sv[j * d + e];
-      else if (j < B + count) v = to_f(wv[(size_t)(j - B) * d + e]);
-      else v = Mh[(size_t)(j - B - count) * d + e];
-      acc += ss[i * ctx + j] * v;
-    }
-    out[(size_t)(b * B + i) * p.nq * d + (size_t)h * d + e] = from_f<T>(acc);
+    out[(size_t)(b * B + i) * p.nq * d + (size_t)h * d + e] = from_f<T>(acc[idx]);
   }
 }
 
@@ -456,7 +516,7 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
       return LSP_ERR_CUDA;
   } else {
     const int ctx = p.B + p.W + p.R;
-    const size_t smem = (size_t)(3 * p.B * p.d + p.B * ctx) * sizeof(float);
+    const size_t smem = (size_t)(3 * p.B * p.d + p.B * ctx + 4 + kSimpleChunk * p.d) * sizeof(float);
     if (smem > 227 * 1024) return LSP_ERR_SHAPE;
     static bool attr32 = false;
     if (!attr32) {
@@ -464,7 +524,7 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
                            227 * 1024);
       attr32 = true;
     }
-    if (launch_pdl(attn_simple_kernel<float>, dim3(p.C * p.nq), dim3(128), smem, s, p) != cudaSuccess)
+    if (launch_pdl(attn_simple_kernel<float>, dim3(p.C * p.nq), dim3(256), smem, s, p) != cudaSuccess)
       return LSP_ERR_CUDA;
   }
   return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;

@@ -4,6 +4,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 
@@ -136,7 +137,7 @@ int lsp_config_check(const lsp_config* c) {
     if (c->d != 128 || c->B > 16 || c->R > 16) return LSP_ERR_SHAPE;
     if (lsp::attn_smem_bytes(c->B, c->W, c->nq, c->nkv) > 227 * 1024) return LSP_ERR_SHAPE;
   } else {
-    if ((size_t)(3 * c->B * c->d + c->B * (c->B + c->W + c->R)) * 4 > 227 * 1024) return LSP_ERR_SHAPE;
+    if ((size_t)(3 * c->B * c->d + c->B * (c->B + c->W + c->R) + 4 + 64 * c->d) * 4 > 227 * 1024) return LSP_ERR_SHAPE;
   }
   for (int j = 0; j < c->D; ++j)
     if (c->layer_map[j] >= c->L) return LSP_ERR_SHAPE;
@@ -166,6 +167,22 @@ static void partial_shapes(const lsp_config& c, int* M, int* K, int* N, int* n) 
   M[i] = Mt; K[i] = c.nq * c.d; N[i++] = c.H;                      // o
   M[i] = Mt; K[i] = c.F; N[i++] = c.H;                             // down
   *n = i;
+}
+
+// Split-K factor of the gate/up projection.  1 (default): one pass with the
+// SwiGLU fused into the GEMM epilogue; > 1 (LSP_GEMM_GU_SPLITS=n): fp32
+// partials [n][M][2F] and a swiglu_sum kernel, which lets the 2F/128 weight
+// tiles fill every SM (the fused form cannot split K: the nonlinearity needs
+// the full sums).  At the Qwen3-8B round the split measured no faster (gate/up
+// 361 us per round with 3 splits, 364 fused; 2 and 4 splits slower) -- each
+// CTA's stream rate, not SM coverage, bounds it -- so fused is the default.
+static int gate_up_splits(const lsp_config& c, int num_sms) {
+  const char* v = std::getenv("LSP_GEMM_GU_SPLITS");
+  if (!v || c.F % kTileRows) return 1;               // the gate and up segments tile separately
+  int splits = std::max(1, std::atoi(v)), wt = 0;
+  const int rows[1] = {2 * c.F};
+  gemm_choose(c.dtype, c.C * c.B, c.H, gemm_tiles(EPI_PARTIAL, rows, 1), EPI_PARTIAL, num_sms, &splits, &wt);
+  return splits;
 }
 
 int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
@@ -220,6 +237,8 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
                 &splits, &wt);
     pbytes = std::max(pbytes, (size_t)splits * pm[i] * pn[i] * sizeof(float));
   }
+  const int gus = gate_up_splits(c, st->num_sms);                   // gate | up, when split
+  if (gus > 1) pbytes = std::max(pbytes, (size_t)gus * M * 2 * c.F * sizeof(float));
   st->nblk = sample_blocks(st->num_sms);
   off = 0;
   const size_t w_x = off; off = align256(off + (size_t)M * c.H * 4);
@@ -393,8 +412,15 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
       return rc;
     const void* Wgu[2] = {lw.w_gate, lw.w_up};
     const int rgu[2] = {c.F, c.F};
-    if ((rc = plan(&st->gu_op[j], st->xn, M, c.H, Wgu, rgu, 2, EPI_SWIGLU, st->act, c.F)) != LSP_OK)
+    const int gus = gate_up_splits(c, st->num_sms);
+    if (gus > 1) {
+      const int r = gemm_plan(&st->gu_op[j], c.dtype, st->xn, M, c.H, Wgu, rgu, 2, EPI_PARTIAL, st->part,
+                              2 * c.F, st->err, st->num_sms, gus, 0);
+      if (r != LSP_OK) return r;
+      if ((size_t)st->gu_op[j].p.out_splits * M * 2 * c.F * sizeof(float) > st->part_bytes) return LSP_ERR_SHAPE;
+    } else if ((rc = plan(&st->gu_op[j], st->xn, M, c.H, Wgu, rgu, 2, EPI_SWIGLU, st->act, c.F)) != LSP_OK) {
       return rc;
+    }
     const void* Wd[1] = {lw.w_down};
     const int rd[1] = {c.H};
     if ((rc = plan(&st->down_op[j], st->act, M, c.F, Wd, rd, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
@@ -478,6 +504,9 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
       return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->gu_op[j], s)) != LSP_OK) return rc;
+    if (st->gu_op[j].p.mode == EPI_PARTIAL &&
+        (rc = launch_swiglu_sum(st->part, st->gu_op[j].p.out_splits, M, c.F, st->act, c.dtype, s)) != LSP_OK)
+      return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->down_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
@@ -549,7 +578,8 @@ int lsp_round_launches(lsp_state* st) {
   // view update, fuse, combine; per layer q/k/v GEMM + finalize, attention, o, norm, gate/up, down,
   // norm; LM head; the sampler
   const int fuse = (c.flags & LSP_NO_BOUNDARY) ? 0 : 1;
-  return 2 + fuse + 8 * c.D + 1 + sample_launches(p, c.dtype);
+  const int gu_sum = gate_up_splits(c, st->num_sms) > 1 ? c.D : 0;   // the swiglu_sum kernels
+  return 2 + fuse + 8 * c.D + gu_sum + 1 + sample_launches(p, c.dtype);
 }
 
 const char* lsp_stage_name(lsp_state* st, int k) {

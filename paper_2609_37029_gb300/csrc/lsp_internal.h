@@ -137,6 +137,9 @@ int launch_combine(const CombineParams& p, int dtype, cudaStream_t s);
 // x += sum_s part[s] (s < splits, fp32 [splits][M][H]); out = RMSNorm(x) * w.
 int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
                       int H, float eps, int dtype, cudaStream_t s);
+// out[m][f] = silu(g) * u with g = sum_s part[s][m][f], u = sum_s part[s][m][F + f]
+// (part fp32 [splits][M][2F]; out dtype [M][F]).
+int launch_swiglu_sum(const float* part, int splits, int M, int F, void* out, int dtype, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention
 // q | k | v of the block rows: sum of the projection's split-K partials, then

@@ -112,6 +112,15 @@ def test_round_with_cluster_split_k(lsp, monkeypatch):
     _run_round(lsp, s, 2500)
 
 
+@pytest.mark.parametrize("gu_splits", ["1", "3"])
+def test_round_gate_up_fused_or_split(lsp, monkeypatch, gu_splits):
+    """The gate/up projection with its SwiGLU fused into the GEMM epilogue (one pass), or
+    split over K with fp32 partials and a separate sum + SwiGLU kernel."""
+    monkeypatch.setenv("LSP_GEMM_GU_SPLITS", gu_splits)
+    s = synth.SMALL
+    _run_round(lsp, s, 1500)
+
+
 def test_round_sampled_and_short_prefix(lsp):
     """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
     s = synth.SMALL.with_(temperature=1.0)
