@@ -70,7 +70,11 @@ __global__ void __launch_bounds__(512)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = blockIdx.x / p.nkv, g = blockIdx.x % p.nkv;
   griddep_launch();
-  griddep_wait();
+  // The window, summary and t come from the view update at the start of the
+  // round: the q/k/v finalize before this kernel triggers its dependents only
+  // after its own wait, so every kernel before the q/k/v projection has
+  // completed and these loads may start before this kernel's own wait,
+  // overlapping the finalize.  Only the block q/k/v waits for it.
   const int B = p.B, L = p.L, l = p.layer;
   const long long t = p.t[b];
   const int count = (int)(t < p.W ? t : p.W);
@@ -124,6 +128,7 @@ __global__ void __launch_bounds__(512)
     const bf16* qkv = static_cast<const bf16*>(p.qkv);
     const int ldq = (p.nq + 2 * p.nkv) * kHD;
     const int kinds = rep + 2;
+    griddep_wait();                                 // the q/k/v finalize has completed
     for (int idx = tid; idx < B * kinds * 16; idx += nthr) {
       const int c = (idx & 15) * 8, item = idx >> 4;
       const int i = item / kinds, kind = item % kinds;
@@ -413,8 +418,11 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
 // its rotary partner lives in lane l ^ 16).
 template <typename T, int EPL>
 __global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
-  griddep_launch();
+  // wait first, then let the attention kernel launch: it reads the view
+  // state before its own wait, which is safe once the q/k/v projection (and
+  // so every kernel before it) has completed
   griddep_wait();
+  griddep_launch();
   const int heads = p.nq + 2 * p.nkv;
   const int item = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;

@@ -617,6 +617,110 @@ __global__ void __launch_bounds__(kPThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------ persistent kernel, fp32 storage
+// One cooperative launch for all B steps with fp32 W_c / E_c (the fp32
+// reference shape): CTA k owns 16-row vocabulary tiles [t_begin, t_begin +
+// cnt) and keeps their W_c rows resident in shared memory.  Per step, a warp
+// takes one request at a time: its lanes form z = z^(0) + W_c[v] . E_c(y)
+// (fp32 FMA) over the slice, write the corrected logits, add the noise and
+// keep a running argmax, which the warp publishes as one 64-bit atomicMax key.
+// Thread 0 then arrives on the step's counter (release) and waits, bounded,
+// for every CTA; y_i is read back from the keys and E_c(y_i) gathered for the
+// next step.  The synchronisation words are those of the bf16 kernel and are
+// left zero at exit.
+constexpr int kPfThreads = 256;
+
+__global__ void __launch_bounds__(kPfThreads, 1)
+    sample_persistent_f32_kernel(const SampleParams p, const int ntiles) {
+  extern __shared__ __align__(16) float pfs[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = kPfThreads / 32;
+  const int nblk = gridDim.x;
+  const int t_begin = (int)(((long long)blockIdx.x * ntiles) / nblk);
+  const int cnt = (int)(((long long)(blockIdx.x + 1) * ntiles) / nblk) - t_begin;
+  const int C = p.C, B = p.B, V = p.V, rc = p.rc;
+  const int v0 = t_begin * 16, nv = cnt * 16;
+  float* Ws = pfs;                                  // [nv][rc]
+  float* Es = Ws + (size_t)nv * rc;                 // [C][rc]
+  __shared__ int s_y[kPMaxC];
+  __shared__ int s_ok;
+  unsigned long long* slots = p.sync;
+  unsigned* counts = reinterpret_cast<unsigned*>(p.sync + (size_t)B * kPMaxC * kSlotStride);
+  const float* Wc = static_cast<const float*>(p.Wc);
+  const float* Ec = static_cast<const float*>(p.Ec);
+  const bool sample = p.temperature > 0.f;
+  const float inv_temp = sample ? 1.0f / p.temperature : 1.0f;
+  const uint2 key = make_uint2((uint32_t)p.seed, (uint32_t)(p.seed >> 32));
+
+  for (int i = tid; i < nv * rc / 4; i += kPfThreads)
+    reinterpret_cast<float4*>(Ws)[i] = reinterpret_cast<const float4*>(Wc + (size_t)v0 * rc)[i];
+  if (tid < C) {
+    int y = p.prev[(size_t)tid * p.prev_stride];
+    if (y < 0 || y >= V) {
+      if (blockIdx.x == 0) set_err(p.err, LSP_DEV_BAD_TOKEN);
+      y = 0;
+    }
+    s_y[tid] = y;
+  }
+  __syncthreads();
+  for (int s = 0; s < B; ++s) {
+    for (int i = tid; i < C * rc; i += kPfThreads) Es[i] = Ec[(size_t)s_y[i / rc] * rc + i % rc];
+    __syncthreads();
+    for (int c = warp; c < C; c += nw) {
+      const float* zr = p.src + ((size_t)c * B + s) * V;
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+      for (int v = v0 + lane; v < v0 + nv; v += 32) {
+        const float* w = Ws + (size_t)(v - v0) * rc;
+        const float* e = Es + (size_t)c * rc;
+        float corr = 0.f;
+        for (int r = 0; r < rc; r += 4) {
+          const float4 a = *reinterpret_cast<const float4*>(w + r), b = *reinterpret_cast<const float4*>(e + r);
+          corr = fmaf(a.x, b.x, corr);
+          corr = fmaf(a.y, b.y, corr);
+          corr = fmaf(a.z, b.z, corr);
+          corr = fmaf(a.w, b.w, corr);
+        }
+        const float z = zr[v] + corr;
+        if (p.dst) p.dst[((size_t)c * B + s) * V + v] = z;
+        float sc = z;
+        if (sample) {
+          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)c, p.round), key);
+          const uint32_t wd = (v & 3) == 0 ? x.x : (v & 3) == 1 ? x.y : (v & 3) == 2 ? x.z : x.w;
+          sc = z * inv_temp + gumbel_of(wd);
+        }
+        if (better(sc, v, bv, bi)) { bv = sc; bi = v; }
+      }
+      unsigned long long k = nv > 0 && bi != 0x7fffffff ? arg_key(bv, bi) : 0ull;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) k = max_u64(k, __shfl_xor_sync(0xffffffffu, k, o));
+      if (lane == 0 && k) atomicMax(&slots[(s * kPMaxC + c) * kSlotStride], k);
+    }
+    __syncthreads();                                // this CTA's keys of step s are published
+    const bool last = s + 1 == B;
+    if (tid == 0) {
+      red_release_add(&counts[s], 1u);
+      s_ok = (last && blockIdx.x != 0) ? 1 : (wait_count(&counts[s], (unsigned)nblk) ? 1 : 0);
+      if (!s_ok) set_err(p.err, LSP_DEV_TIMEOUT);
+    }
+    __syncthreads();
+    if (!s_ok || (last && blockIdx.x != 0)) return;   // only CTA 0 needs y_B
+    if (tid < C) {
+      int y = (int)~(uint32_t)ld_relaxed_u64(&slots[(s * kPMaxC + tid) * kSlotStride]);
+      if (y < 0 || y >= V) {                          // no key arrived: corrupt sync words
+        set_err(p.err, LSP_DEV_TIMEOUT);
+        y = 0;
+      }
+      s_y[tid] = y;
+      if (blockIdx.x == 0) p.out_tokens[(size_t)tid * B + s] = y;
+    }
+    __syncthreads();
+  }
+  // CTA 0 after the last step: every CTA has arrived on every counter, so no
+  // one reads the sync words again -- leave them zero for the next launch
+  for (int i = tid; i < B * kPMaxC; i += kPfThreads) slots[i * kSlotStride] = 0ull;
+  for (int i = tid; i < B; i += kPfThreads) counts[i] = 0u;
+}
+
 __global__ void __launch_bounds__(kSampThreads) sample_final_kernel(const SampleParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   griddep_launch();
@@ -703,6 +807,55 @@ static int launch_persistent(const SampleParams& p, cudaStream_t s) {
 }
 
 // The persistent kernel's shape limits (anything else takes the per-step kernel).
+static size_t persistent_f32_smem(int tpc, int rc) { return ((size_t)tpc * 16 + kPMaxC) * rc * sizeof(float); }
+
+static bool coop_ok() {
+  int dev = 0, coop = 0;
+  return cudaGetDevice(&dev) == cudaSuccess &&
+         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop != 0;
+}
+
+// fp32 storage: the whole B-step loop in one cooperative launch when the W_c
+// slice of a CTA fits shared memory.
+static bool persistent_f32_ok(const SampleParams& p, int dtype) {
+  if (dtype != LSP_DTYPE_F32 || p.C > kPMaxC || !p.sync || p.num_sms < 1 || p.rc % 4) return false;
+  const int ntiles = p.V / 16;
+  const int nblk = std::min(p.num_sms, ntiles);
+  const int tpc = (ntiles + nblk - 1) / nblk;
+  return persistent_f32_smem(tpc, p.rc) <= 200 * 1024 && coop_ok();
+}
+
+static int launch_persistent_f32(const SampleParams& p, cudaStream_t s) {
+  const int ntiles = p.V / 16;
+  const int nblk = std::min(p.num_sms, ntiles);
+  const int tpc = (ntiles + nblk - 1) / nblk;
+  const size_t smem = persistent_f32_smem(tpc, p.rc);
+  static size_t attr = 0;
+  if (smem > attr) {
+    if (cudaFuncSetAttribute(sample_persistent_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem) != cudaSuccess)
+      return LSP_ERR_CUDA;
+    attr = smem;
+  }
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sample_persistent_f32_kernel, kPfThreads,
+                                                    smem) != cudaSuccess)
+    return LSP_ERR_CUDA;
+  if (per_sm < 1) return LSP_ERR_SHAPE;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(nblk);
+  cfg.blockDim = dim3(kPfThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr_c[1];
+  attr_c[0].id = cudaLaunchAttributeCooperative;       // every CTA resident: the step waits are safe
+  attr_c[0].val.cooperative = 1;
+  cfg.attrs = attr_c;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sample_persistent_f32_kernel, p, ntiles) == cudaSuccess ? LSP_OK
+                                                                                         : LSP_ERR_CUDA;
+}
+
 static bool persistent_ok(const SampleParams& p, int dtype) {
   if (dtype != LSP_DTYPE_BF16 || p.C > kPMaxC || (p.rc != 32 && p.rc != 64) || !p.sync || p.num_sms < 1)
     return false;
@@ -710,14 +863,12 @@ static bool persistent_ok(const SampleParams& p, int dtype) {
   const int nblk = std::min(p.num_sms, ntiles);
   const int tpc = (ntiles + nblk - 1) / nblk;
   if (tpc > kPMaxTiles || persistent_smem(tpc, p.rc) > 227 * 1024) return false;
-  int dev = 0, coop = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess)
-    return false;
-  return coop != 0;
+  return coop_ok();
 }
 
-int sample_launches(const SampleParams& p, int dtype) { return persistent_ok(p, dtype) ? 1 : p.B + 1; }
+int sample_launches(const SampleParams& p, int dtype) {
+  return persistent_ok(p, dtype) || persistent_f32_ok(p, dtype) ? 1 : p.B + 1;
+}
 
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if (p.C > kMaxC || p.V % 16 || p.rc % 16 || p.rc > 256) return LSP_ERR_SHAPE;
@@ -727,6 +878,7 @@ int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
     return LSP_ERR_ARG;
   if (persistent_ok(p, dtype))
     return p.rc == 32 ? launch_persistent<2>(p, s) : launch_persistent<4>(p, s);
+  if (persistent_f32_ok(p, dtype)) return launch_persistent_f32(p, s);
 
   if (p.nblk > 32 * kMaxPartialsPerLane) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
