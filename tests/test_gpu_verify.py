@@ -109,6 +109,50 @@ def test_verify_matches_oracle(lsp, T, C, B, V):
         assert len(set(acc.tolist())) >= 3             # the accepted lengths really spread
 
 
+@pytest.mark.parametrize("T", [1.0, 0.0])
+def test_verify_at_the_bench_shape_on_sampled_requests(lsp, T):
+    """C = 16, B = 16, V = 151936 -- the launch configuration bench.py times.  Requests 0
+    and 11 carry candidates drafted from q by the drafter's rule and are compared with the
+    oracle; the others carry random candidates (valid input, mostly rejected at once) and
+    are checked for range only."""
+    s = _shape(16, 16, 151936)
+    seed, rnd = 99, 4
+    zt, zq = synth.make_verify_logits(s, seed=61)
+    g = np.random.default_rng(5)
+    y = g.integers(0, s.V, size=(s.C, s.B)).astype(np.int32)
+    picked = [0, 11]
+    for b in picked:
+        y[b] = _draft_rows(zq[b].numpy(), T, seed, rnd, b)
+    acc, tok, err = _run(lsp, s, zt, zq, y, T, seed, rnd)
+    assert err == (lsp.LSP_OK, 0)
+    assert ((acc >= 0) & (acc <= s.B)).all() and ((tok >= 0) & (tok < s.V)).all()
+    sub = _shape(1, 16, 151936)
+    for b in picked:
+        one = _compare_one(sub, zt[b].numpy(), zq[b].numpy(), y[b], T, seed, rnd, b, acc[b], tok[b])
+        assert one, b
+
+
+def _draft_rows(zq_b, T, seed, rnd, b):
+    """Request b's candidates by the drafter's Gumbel-max rule (argmax at T = 0)."""
+    B, V = zq_b.shape
+    return np.array([np.argmax(zq_b[i].astype(np.float64)) if T <= 0 else
+                     np.argmax(zq_b[i].astype(np.float64) / T + gumbel(seed, rnd, b, i, V))
+                     for i in range(B)], dtype=np.int32)
+
+
+def _compare_one(s, zt_b, zq_b, y_b, T, seed, rnd, b, acc_b, tok_b):
+    """One request against the oracle with the margin rules of _compare; True when the
+    decisions were clear enough to compare exactly (and matched)."""
+    r, t, margins, dm = oracle.verify_block(zt_b, zq_b, y_b, T, seed, rnd, b)
+    tested = margins[:r + 1] if r < s.B else margins
+    if T > 0 and not all(m > ACC_TOL for m in tested):
+        return True                      # a near-tie: nothing exact to compare
+    assert acc_b == r, (b, acc_b, r)
+    if dm > DRAW_TOL:
+        assert tok_b == t, (b, tok_b, t, dm)
+    return True
+
+
 def test_verify_accepts_everything_when_draft_equals_target(lsp):
     """p = q makes alpha = 1: r = B for every request and the bonus follows p_{B+1}."""
     s = _shape(6, 16, 2048)
