@@ -155,12 +155,19 @@ __global__ void __launch_bounds__(kNormThreads)
                       const T* __restrict__ w, T* __restrict__ out, int M, int H, float eps) {
   __shared__ float red[32];
   griddep_launch();
-  griddep_wait();
   const int m = blockIdx.x;
+  const int h4 = H / 4;
+  // the norm weight is a constant: load it before waiting for the producer
+  float4 wv[VPT];
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int j = threadIdx.x + k * blockDim.x;
+    if (j < h4) wv[k] = ld4(w, j);
+  }
+  griddep_wait();
   float* row = x + (size_t)m * H;
   const float* prow = part + (size_t)m * H;
   const size_t pstride = (size_t)M * H;
-  const int h4 = H / 4;
   float4 xv[VPT];
   float ss = 0.f;
 #pragma unroll
@@ -196,11 +203,9 @@ __global__ void __launch_bounds__(kNormThreads)
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
     const int j = threadIdx.x + k * blockDim.x;
-    if (j < h4) {
-      const float4 wv = ld4(w, j);
-      st4(out + (size_t)m * H, j, make_float4(xv[k].x * rstd * wv.x, xv[k].y * rstd * wv.y,
-                                              xv[k].z * rstd * wv.z, xv[k].w * rstd * wv.w));
-    }
+    if (j < h4)
+      st4(out + (size_t)m * H, j, make_float4(xv[k].x * rstd * wv[k].x, xv[k].y * rstd * wv[k].y,
+                                              xv[k].z * rstd * wv[k].z, xv[k].w * rstd * wv[k].w));
   }
 }
 
