@@ -47,6 +47,11 @@ template <> struct GemmType<float> {
 
 constexpr uint32_t kTileBytes = kTileRows * 128;   // one weight tile per stage: 16 KB
 
+// The epilogue's named barrier (id 1) counts exactly the four epilogue warps
+// 2-5: any other warp taking that branch would leave bar.sync waiting forever.
+constexpr int kEpilogueThreads = 128;
+static_assert(kGemmThreads == 64 + kEpilogueThreads, "warp 0 TMA, warp 1 MMA, warps 2-5 epilogue");
+
 // Instruction descriptor: fp32 accumulate, A/B format `fmt`, both K-major,
 // N = n, M = 128.
 __device__ __forceinline__ uint32_t make_idesc(int n, uint32_t fmt) {
@@ -61,7 +66,7 @@ __device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int sp
   if (p.mode == EPI_SWIGLU) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) xchg[r * 17 + j] = v[j];
-    named_bar(1, 128);
+    named_bar(1, kEpilogueThreads);
     if (r < 64) {
       const int f = tile * 64 + r;
       T* Y = static_cast<T*>(p.Y);
@@ -75,7 +80,7 @@ __device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int sp
         }
       }
     }
-    named_bar(1, 128);
+    named_bar(1, kEpilogueThreads);
     return;
   }
   const int n = tile * kTileRows + r;
@@ -126,12 +131,12 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
       else tmem_ld16(lane_base + col, v);
       uint8_t* stg = stg0 + (chunk & 1) * buf_bytes;
       if (issuer && chunk >= 2) bulk_wait_read<1>();         // the store two chunks back has read stg
-      named_bar(1, 128);
+      named_bar(1, kEpilogueThreads);
       if (swiglu) {
 #pragma unroll
         for (int j = 0; j < 32; ++j)
           if (j < TT) xchg[r * kXchgStride + j] = v[j];
-        named_bar(1, 128);
+        named_bar(1, kEpilogueThreads);
         // thread (f = r & 63, half = r >> 6) forms tokens [half * TT/2, (half + 1) * TT/2)
         const int f = r & 63, t0 = (r >> 6) * (TT / 2);
         T* o = reinterpret_cast<T*>(stg);
@@ -155,7 +160,7 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
           if (j < TT) o[j * kTileRows + r] = from_f<T>(v[j]);
       }
       fence_proxy_async_smem();
-      named_bar(1, 128);
+      named_bar(1, kEpilogueThreads);
       if (issuer) {
         tma_store_3d(to, smem_u32(stg), (tile0 + w) * cols, m0, split);
         bulk_commit();
@@ -399,7 +404,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const bool ok = mbar_wait(acc_bar, 0, p.err);
     if (!ok) *s_abort = 1;
     tc_fence_after();
-    named_bar(1, 128);
+    named_bar(1, kEpilogueThreads);
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
     if (p.creduce) {
       // reduced across the cluster below, by the whole CTA
