@@ -11,10 +11,16 @@
 // last CTA of each request advances t.
 //
 // One CTA per (request b, tapped layer l, KV head g) covers the nq/nkv query
-// heads sharing that KV head (rep * R queries): the new K/V rows are read from
-// HBM once (16-byte vectors) and staged in shared memory as fp32; each warp
-// owns whole queries, lanes split the head dimension, and the dot products and
-// the row max/sum reduce with warp shuffles.  Only the new rows are touched.
+// heads sharing that KV head (rep * R queries); the new K/V rows are read from
+// HBM once (16-byte vectors) and only the new rows are touched.
+// view_update_mma_kernel (bf16, d = 128, rep * R in {16, 32, 64}): the
+// statistics are an attention of the summary queries over the new rows, run
+// as mma.sync tiles with an online softmax (below).  view_update_kernel (every
+// other shape): rows staged in shared memory as fp32; each warp owns whole
+// queries, lanes split the head dimension, and the dot products and the row
+// max/sum reduce with warp shuffles.
+#include <cstdlib>
+
 #include "common.cuh"
 #include "lsp_internal.h"
 
@@ -208,6 +214,244 @@ __global__ void __launch_bounds__(kViewThreads)
   }
 }
 
+// ---------------------------------------------------------------- tensor-core variant
+// bf16 storage, d = 128, Q = rep * R in {16, 32, 64}: the summary update is
+// the attention of the Q summary queries over the new rows, so it runs as
+// mma.sync m16n8k16 tiles.  Warp w owns query tile w % MT (16 queries) and
+// head dims [(w / MT) * 8 * NT, +8 NT): per 16-row key chunk S = G K^T (bf16
+// products are exact, fp32 accumulate), an online softmax in registers, and
+// P V with P split into a bf16 high part and the bf16 remainder (two MMAs:
+// ~16 significant bits of every weight).  The stored (eta, m) stay in the
+// accumulator layout in registers from the first load to the final store.
+constexpr int kVuRows = 64;                // new rows staged per pass
+constexpr int kVuLd = 128 + 8;             // smem row (bf16): conflict-free ldmatrix
+
+template <int MT>
+__global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const ViewParams p) {
+  constexpr int NT = 16 * MT / kViewWarps;                 // 8-dim output tiles per warp
+  constexpr int Q = 16 * MT;
+  extern __shared__ __align__(16) uint8_t vsm_raw[];
+  bf16* sG = reinterpret_cast<bf16*>(vsm_raw);             // [Q][kVuLd]
+  bf16* sK = sG + Q * kVuLd;                               // [kVuRows][kVuLd]
+  bf16* sV = sK + kVuRows * kVuLd;
+  constexpr int d = 128;
+  const int unit = blockIdx.x;
+  const int g = unit % p.nkv;
+  const int l = (unit / p.nkv) % p.L;
+  const int b = unit / (p.nkv * p.L);
+  const int rep = p.nq / p.nkv;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int mt = warp % MT, d0 = (warp / MT) * 8 * NT;     // this warp's query tile and first dim
+  griddep_launch();
+  // the summary queries are a constant of the state: stage them before the wait
+  const size_t gbase = ((size_t)l * p.nq + (size_t)g * rep) * p.R;
+  const bf16* Gp = static_cast<const bf16*>(p.G) + gbase * d;
+  for (int i = tid; i < Q * 16; i += kViewThreads) {
+    const int q = i >> 4, c = (i & 15) * 8;
+    cp_async16(sG + q * kVuLd + c, Gp + (size_t)q * d + c);
+  }
+  griddep_wait();
+
+  const int delta = p.acc[b];
+  if (delta < 0 || delta > p.rows) {
+    if (tid == 0 && g == 0 && l == 0) set_err(p.err, LSP_DEV_BAD_DELTA);
+    cp_async_wait_all();
+    return;
+  }
+  if (delta == 0) { cp_async_wait_all(); return; }        // empty new set: state unchanged (App. A.2)
+  const long long t0 = p.t[b];
+
+  // ---- the stored state of this warp's rows (r0, r0 + 8) and dims, accumulator layout
+  const size_t qbase = ((size_t)(b * p.L + l) * p.nq + (size_t)g * rep) * p.R;
+  const int r0 = mt * 16 + (lane >> 2);
+  float* mA = p.m + (qbase + r0) * d + d0 + (lane & 3) * 2;
+  float acc[NT][4];
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+    const float2 x0 = *reinterpret_cast<const float2*>(mA + n * 8);
+    const float2 x1 = *reinterpret_cast<const float2*>(mA + 8 * d + n * 8);
+    acc[n][0] = x0.x; acc[n][1] = x0.y; acc[n][2] = x1.x; acc[n][3] = x1.y;
+  }
+  const float etaA0 = p.eta[qbase + r0], etaA1 = p.eta[qbase + r0 + 8];
+  cp_async_wait_all();
+  __syncthreads();
+  // A operand (G rows of this warp's tile) for the 8 k-steps, kept in registers
+  uint32_t ga[8][4];
+  {
+    const bf16* qa = sG + (size_t)(mt * 16 + (lane & 15)) * kVuLd + (lane >> 4) * 8;
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) ldsm_x4(ga[kk], qa + kk * 16);
+  }
+
+  const float sl2 = 1.4426950408889634f * rsqrtf((float)d);   // log2(e) / sqrt(d)
+  float rmax[2] = {-INFINITY, -INFINITY}, rsum[2] = {0.f, 0.f};
+  float o[NT][4];
+#pragma unroll
+  for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+
+  const bf16* kin = static_cast<const bf16*>(p.k_new);
+  const bf16* vin = static_cast<const bf16*>(p.v_new);
+  bf16* wk = static_cast<bf16*>(p.win_k);
+  bf16* wv = static_cast<bf16*>(p.win_v);
+  const size_t row_stride = (size_t)p.nkv * d;
+  const size_t in_base = (size_t)(b * p.L + l) * p.rows * row_stride + (size_t)g * d;
+  const size_t win_base = ((size_t)(b * p.L + l) * p.nkv + g) * (size_t)p.W * d;
+
+  for (int j0 = 0; j0 < delta; j0 += kVuRows) {
+    const int nrows = min(kVuRows, delta - j0);
+    const int nrows16 = (nrows + 15) / 16 * 16;
+    __syncthreads();                                       // previous rows consumed
+    // stage K and V rows (zero past nrows) and write the window ring
+    for (int idx = tid; idx < 2 * nrows16 * 16; idx += kViewThreads) {
+      const int which = idx / (nrows16 * 16), rem = idx % (nrows16 * 16);
+      const int j = rem >> 4, c = (rem & 15) * 8;
+      uint4 raw = make_uint4(0u, 0u, 0u, 0u);
+      if (j < nrows) {
+        raw = *reinterpret_cast<const uint4*>((which ? vin : kin) + in_base + (size_t)(j0 + j) * row_stride + c);
+        if (p.W > 0 && j0 + j >= delta - p.W) {
+          const long long pabs = t0 + j0 + j;
+          *reinterpret_cast<uint4*>((which ? wv : wk) + win_base + (size_t)(pabs % p.W) * d + c) = raw;
+        }
+      }
+      *reinterpret_cast<uint4*>((which ? sV : sK) + j * kVuLd + c) = raw;
+    }
+    __syncthreads();
+    for (int c16 = 0; c16 < nrows16; c16 += 16) {
+      // S = G K^T over 16 keys: two n8 tiles
+      float sc[2][4];
+#pragma unroll
+      for (int n = 0; n < 2; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+      const bf16* kb = sK + (size_t)(c16 + (lane & 7) + (lane >> 4) * 8) * kVuLd + ((lane >> 3) & 1) * 8;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        uint32_t bk[4];
+        ldsm_x4(bk, kb + kk * 16);
+        mma_bf16(sc[0], ga[kk], bk[0], bk[1]);
+        mma_bf16(sc[1], ga[kk], bk[2], bk[3]);
+      }
+      const int nvalid = nrows - c16;
+#pragma unroll
+      for (int n = 0; n < 2; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (n * 8 + (lane & 3) * 2 + (e & 1) >= nvalid) sc[n][e] = -INFINITY;
+      float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][1]), fmaxf(sc[1][0], sc[1][1]));
+      float mx1 = fmaxf(fmaxf(sc[0][2], sc[0][3]), fmaxf(sc[1][2], sc[1][3]));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float n0 = fmaxf(rmax[0], mx0), n1 = fmaxf(rmax[1], mx1);   // finite: key 0 of a chunk is valid
+      const float s0 = exp2f((rmax[0] - n0) * sl2), s1 = exp2f((rmax[1] - n1) * sl2);
+      rmax[0] = n0;
+      rmax[1] = n1;
+      float pr[2][4];
+#pragma unroll
+      for (int n = 0; n < 2; ++n) {
+        pr[n][0] = exp2f((sc[n][0] - n0) * sl2);
+        pr[n][1] = exp2f((sc[n][1] - n0) * sl2);
+        pr[n][2] = exp2f((sc[n][2] - n1) * sl2);
+        pr[n][3] = exp2f((sc[n][3] - n1) * sl2);
+      }
+      rsum[0] = rsum[0] * s0 + pr[0][0] + pr[0][1] + pr[1][0] + pr[1][1];
+      rsum[1] = rsum[1] * s1 + pr[0][2] + pr[0][3] + pr[1][2] + pr[1][3];
+#pragma unroll
+      for (int n = 0; n < NT; ++n) {
+        o[n][0] *= s0; o[n][1] *= s0;
+        o[n][2] *= s1; o[n][3] *= s1;
+      }
+      // P = high + remainder, both bf16
+      uint32_t ph[4], pl[4];
+      {
+        const float q00 = pr[0][0], q01 = pr[0][1], q02 = pr[0][2], q03 = pr[0][3];
+        const float q10 = pr[1][0], q11 = pr[1][1], q12 = pr[1][2], q13 = pr[1][3];
+        ph[0] = pack_bf16(q00, q01); ph[1] = pack_bf16(q02, q03);
+        ph[2] = pack_bf16(q10, q11); ph[3] = pack_bf16(q12, q13);
+        auto rem_of = [](float x) { return x - __bfloat162float(__float2bfloat16_rn(x)); };
+        pl[0] = pack_bf16(rem_of(q00), rem_of(q01)); pl[1] = pack_bf16(rem_of(q02), rem_of(q03));
+        pl[2] = pack_bf16(rem_of(q10), rem_of(q11)); pl[3] = pack_bf16(rem_of(q12), rem_of(q13));
+      }
+      const bf16* vb = sV + (size_t)(c16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kVuLd + d0 + (lane >> 4) * 8;
+#pragma unroll
+      for (int np = 0; np < NT / 2; ++np) {
+        uint32_t bv[4];
+        ldsm_x4_t(bv, vb + np * 16);
+        mma_bf16(o[2 * np], ph, bv[0], bv[1]);
+        mma_bf16(o[2 * np + 1], ph, bv[2], bv[3]);
+        mma_bf16(o[2 * np], pl, bv[0], bv[1]);
+        mma_bf16(o[2 * np + 1], pl, bv[2], bv[3]);
+      }
+    }
+  }
+  rsum[0] += __shfl_xor_sync(0xffffffffu, rsum[0], 1);
+  rsum[0] += __shfl_xor_sync(0xffffffffu, rsum[0], 2);
+  rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 1);
+  rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 2);
+
+  // ---- (eta_N, m_N) of the new rows, merged into (eta_A, m_A) by Eq. summary-update
+  const float isd = rsqrtf((float)d);
+  const float etaN[2] = {rmax[0] * isd + logf(rsum[0]), rmax[1] * isd + logf(rsum[1])};
+  const float etaA[2] = {etaA0, etaA1};
+  float ca[2], cn[2], eta[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const float mx = fmaxf(etaA[h], etaN[h]);
+    eta[h] = mx + logf(__expf(etaA[h] - mx) + __expf(etaN[h] - mx));
+    ca[h] = __expf(etaA[h] - eta[h]);
+    cn[h] = __expf(etaN[h] - eta[h]) / rsum[h];            // m_N = o / rsum
+  }
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+    const float2 y0 = make_float2(ca[0] * acc[n][0] + cn[0] * o[n][0], ca[0] * acc[n][1] + cn[0] * o[n][1]);
+    const float2 y1 = make_float2(ca[1] * acc[n][2] + cn[1] * o[n][2], ca[1] * acc[n][3] + cn[1] * o[n][3]);
+    *reinterpret_cast<float2*>(mA + n * 8) = y0;
+    *reinterpret_cast<float2*>(mA + 8 * d + n * 8) = y1;
+  }
+  if (d0 == 0 && (lane & 3) == 0) {
+    p.eta[qbase + r0] = eta[0];
+    p.eta[qbase + r0 + 8] = eta[1];
+  }
+
+  // ---- boundary: hidden state of the last new row, this CTA's 1/nkv share
+  if (p.h) {
+    const bf16* hin = static_cast<const bf16*>(p.h_new) + ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
+    bf16* hout = static_cast<bf16*>(p.h) + (size_t)(b * p.L + l) * p.H;
+    const int per = p.H / p.nkv;
+    for (int i = g * per + tid * 8; i < (g + 1) * per; i += kViewThreads * 8)
+      *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
+  }
+  // ---- the last CTA of request b advances t
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const int old = atomicAdd(&p.done[b], 1);
+    if (old == p.L * p.nkv - 1) {
+      p.t[b] = t0 + delta;
+      p.done[b] = 0;
+      __threadfence();
+    }
+  }
+}
+
+// LSP_VIEW_FMA=1 keeps the FMA kernel (for measurement)
+static bool view_mma_enabled() { return std::getenv("LSP_VIEW_FMA") == nullptr; }
+
+template <int MT>
+static int launch_mma(const ViewParams& p, cudaStream_t s) {
+  const size_t smem = (size_t)(16 * MT + 2 * kVuRows) * kVuLd * sizeof(bf16);
+  static size_t attr = 0;
+  if (smem > attr) {
+    if (cudaFuncSetAttribute(view_update_mma_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
+      return LSP_ERR_CUDA;
+    attr = smem;
+  }
+  return launch_pdl(view_update_mma_kernel<MT>, dim3(p.C * p.L * p.nkv), dim3(kViewThreads), smem, s, p) ==
+                 cudaSuccess
+             ? LSP_OK
+             : LSP_ERR_CUDA;
+}
+
 template <typename T, int DPL>
 static int launch_dpl(const ViewParams& p, cudaStream_t s) {
   const int Q = (p.nq / p.nkv) * p.R;
@@ -227,6 +471,13 @@ static int launch_dpl(const ViewParams& p, cudaStream_t s) {
 }
 
 int launch_view_update(const ViewParams& p, int dtype, cudaStream_t s) {
+  // tensor-core path: bf16, d = 128, Q = rep * R a power of two from 16 to 64
+  const int Q = (p.nq / p.nkv) * p.R;
+  if (dtype == LSP_DTYPE_BF16 && p.d == 128 && view_mma_enabled()) {
+    if (Q == 64) return launch_mma<4>(p, s);
+    if (Q == 32) return launch_mma<2>(p, s);
+    if (Q == 16) return launch_mma<1>(p, s);
+  }
   if (p.d == 128) return dtype == LSP_DTYPE_BF16 ? launch_dpl<bf16, 4>(p, s) : launch_dpl<float, 4>(p, s);
   if (p.d == 64) return dtype == LSP_DTYPE_BF16 ? launch_dpl<bf16, 2>(p, s) : launch_dpl<float, 2>(p, s);
   return LSP_ERR_SHAPE;
