@@ -375,6 +375,20 @@ class Workload:
         return g
 
 
+def round_percentiles(g, n=200):
+    """Per-round device times of n replays, each between its own pair of CUDA
+    events (after the main timed region): median, p10, p90 in µs."""
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    torch.cuda.synchronize()
+    evs[0].record()
+    for i in range(n):
+        g.replay()
+        evs[i + 1].record()
+    torch.cuda.synchronize()
+    t = sorted(evs[i].elapsed_time(evs[i + 1]) * 1e3 for i in range(n))
+    return {"median": t[n // 2], "p10": t[n // 10], "p90": t[(9 * n) // 10], "n": n}
+
+
 def time_graph(g, steps, warmup, dist, clocks=None):
     if clocks:
         clocks.start()                  # samples span the warm-up and the timed replays
@@ -553,6 +567,7 @@ def run_ours(args, dist):
         raise RuntimeError(f"device error after warm-up: {rc} bits={bits}")
     g = wl.capture(st)
     ms, clocks = time_graph(g, args.steps, args.warmup, dist, Clocks())
+    round_us = round_percentiles(g)
     ms = dist.max(ms)
     rc, bits = lsp.lsp_get_error(st)
     if rc != lsp.LSP_OK:
@@ -657,6 +672,7 @@ def run_ours(args, dist):
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "us_per_round": ms * 1e3,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
+           "round_us": round_us,
            "data": "synthetic (seeded random features and random-init weights)",
            "config": workload_config(s, prefix),
            "roofline": roofline, "round_roofline": round_roof,
