@@ -4,6 +4,7 @@ exactly as the paper's fixed-size interface (Sec. 2.4 "Fixed-cost complexity")."
 import os
 import re
 import subprocess
+import sys
 
 import pytest
 
@@ -76,3 +77,31 @@ def test_bad_layer_map_and_null_args(lsp):
     assert lsp._f["lsp_draft"](None, None, None, None, None, None, None) == lsp.LSP_ERR_ARG
     assert lsp._f["lsp_view_update"](None, None, None, None) == lsp.LSP_ERR_ARG
     assert lsp.lsp_status_string(lsp.LSP_ERR_TIMEOUT) == "device wait timed out"
+
+
+def test_the_binding_refuses_to_run_without_its_library(tmp_path):
+    """No fallback: a copy of the package without liblsp.so fails at import, loudly."""
+    pkg = tmp_path / "paper_2609_37029_gb300"
+    pkg.mkdir()
+    for name in ("__init__.py", "lsp.py", "synth.py"):
+        (pkg / name).write_text(open(os.path.join(ROOT, "paper_2609_37029_gb300", name)).read())
+    r = subprocess.run([sys.executable, "-c", "import paper_2609_37029_gb300.lsp"], cwd=tmp_path,
+                       capture_output=True, text=True, env={**os.environ, "PYTHONPATH": str(tmp_path)})
+    assert r.returncode != 0
+    assert "ImportError" in r.stderr and "liblsp.so" in r.stderr
+
+
+def test_ablation_configs_on_the_host(lsp):
+    """W = 0, R = 0 and LSP_NO_BOUNDARY are valid configs whose interface drops exactly the
+    removed source's bytes; unknown flag bits are rejected."""
+    s = synth.Q8B
+    full = lsp.lsp_state_bytes(lsp.make_config(s))
+    for variant in ({"W": 0}, {"R": 0}, {"no_boundary": True}):
+        v = s.with_(**variant)
+        cfg = lsp.make_config(v)
+        assert lsp.lsp_config_check(cfg) == lsp.LSP_OK
+        assert lsp.lsp_state_bytes(cfg) == s.C * oracle.state_bytes_per_request(v) + 8 * s.C
+    assert lsp.lsp_state_bytes(lsp.make_config(s.with_(no_boundary=True))) == full - s.C * s.L * s.H * 2
+    cfg = lsp.make_config(s)
+    cfg.flags = 2
+    assert lsp.lsp_config_check(cfg) == lsp.LSP_ERR_ARG
