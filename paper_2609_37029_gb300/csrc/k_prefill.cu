@@ -24,6 +24,7 @@
 // e^(eta_s - eta) m_s) -- deterministic -- and writes (eta, m) into the state;
 // further CTAs copy the window rows and the boundary hidden state and set t.
 #include <algorithm>
+#include <cstdlib>
 
 #include "common.cuh"
 #include "lsp_internal.h"
@@ -32,16 +33,20 @@ namespace lsp {
 
 constexpr int kPfD = 128;                 // head dim of this path
 constexpr int kPfLd = kPfD + 8;           // smem row stride (bf16): conflict-free ldmatrix
-constexpr int kPfChunk = 64;              // K/V rows per pipeline stage
+constexpr int kPfChunk = 64;              // segment granularity (a multiple of every stage size)
 constexpr int kPfRec = 16 + 16 * kPfD;    // floats per (segment, layer, query head): eta[16], m[16][d]
+constexpr int kPrefillStage = 32;         // default K/V rows per pipeline stage (measured: 745 vs 897 us at 64)
 
+// CH = K/V rows per pipeline stage (32 or 64): smaller stages leave room for
+// more CTAs per SM (shared memory and registers) at the same MMA work.
+template <int CH>
 __global__ void __launch_bounds__(256)
     prefill_partial_kernel(const PrefillParams p, const int rep, const int seg_rows) {
   extern __shared__ __align__(16) uint8_t psm[];
   const size_t row = kPfLd;
   bf16* sG = reinterpret_cast<bf16*>(psm);                   // [rep * 16][kPfLd]
-  bf16* sK = sG + (size_t)rep * 16 * row;                    // [2][kPfChunk][kPfLd]
-  bf16* sV = sK + (size_t)2 * kPfChunk * row;                // [2][kPfChunk][kPfLd]
+  bf16* sK = sG + (size_t)rep * 16 * row;                    // [2][CH][kPfLd]
+  bf16* sV = sK + (size_t)2 * CH * row;                      // [2][CH][kPfLd]
 
   const int nthr = rep * 32;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -50,7 +55,7 @@ __global__ void __launch_bounds__(256)
   const int r_begin = seg * seg_rows;
   const int r_end = min(p.rows, r_begin + seg_rows);
   const int nrows = r_end - r_begin;
-  const int nchunks = (nrows + kPfChunk - 1) / kPfChunk;
+  const int nchunks = (nrows + CH - 1) / CH;
   griddep_launch();
   griddep_wait();
 
@@ -62,17 +67,17 @@ __global__ void __launch_bounds__(256)
     if (r < p.R) cp_async16(dq, Gp + ((size_t)hh * p.R + r) * kPfD + c8);
     else *reinterpret_cast<uint4*>(dq) = make_uint4(0, 0, 0, 0);
   }
-  // ---- one 64-row chunk of this segment's K/V into buffer `buf`; rows past the
+  // ---- one CH-row chunk of this segment's K/V into buffer `buf`; rows past the
   // segment are zero (their scores are masked and their value rows add nothing)
   const bf16* kin = static_cast<const bf16*>(p.k) + (size_t)l * p.rows * p.nkv * kPfD + (size_t)g * kPfD;
   const bf16* vin = static_cast<const bf16*>(p.v) + (size_t)l * p.rows * p.nkv * kPfD + (size_t)g * kPfD;
   const size_t rstride = (size_t)p.nkv * kPfD;
   auto stage = [&](int c, int buf) {
-    for (int idx = tid; idx < kPfChunk * 16; idx += nthr) {
+    for (int idx = tid; idx < CH * 16; idx += nthr) {
       const int j = idx >> 4, c8 = (idx & 15) * 8;
-      const int rr = r_begin + c * kPfChunk + j;
-      bf16* dk = sK + ((size_t)buf * kPfChunk + j) * row + c8;
-      bf16* dv = sV + ((size_t)buf * kPfChunk + j) * row + c8;
+      const int rr = r_begin + c * CH + j;
+      bf16* dk = sK + ((size_t)buf * CH + j) * row + c8;
+      bf16* dv = sV + ((size_t)buf * CH + j) * row + c8;
       if (rr < r_end) {
         cp_async16(dk, kin + (size_t)rr * rstride + c8);
         cp_async16(dv, vin + (size_t)rr * rstride + c8);
@@ -99,19 +104,20 @@ __global__ void __launch_bounds__(256)
     const int buf = c & 1;
     asm volatile("cp.async.wait_group 1;" ::: "memory");      // chunk c has landed
     __syncthreads();
-    const bf16* Kc = sK + (size_t)buf * kPfChunk * row;
-    const bf16* Vc = sV + (size_t)buf * kPfChunk * row;
-    const int nvalid = min(kPfChunk, nrows - c * kPfChunk);
-    // scores of the warp's 16 queries against the 64 rows: s[n] covers keys 8n..8n+7
-    float s[8][4];
+    const bf16* Kc = sK + (size_t)buf * CH * row;
+    const bf16* Vc = sV + (size_t)buf * CH * row;
+    const int nvalid = min(CH, nrows - c * CH);
+    // scores of the warp's 16 queries against the CH rows: s[n] covers keys 8n..8n+7
+    constexpr int NS = CH / 8;
+    float s[NS][4];
 #pragma unroll
-    for (int n = 0; n < 8; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+    for (int n = 0; n < NS; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < kPfD / 16; ++kk) {
       uint32_t a[4];
       ldsm_x4(a, qbase + kk * 16);
 #pragma unroll
-      for (int nt = 0; nt < 4; ++nt) {
+      for (int nt = 0; nt < CH / 16; ++nt) {
         uint32_t bk[4];
         ldsm_x4(bk, Kc + (size_t)(nt * 16 + (lane & 7) + (lane >> 4) * 8) * row + ((lane >> 3) & 1) * 8 + kk * 16);
         mma_bf16(s[2 * nt], a, bk[0], bk[1]);
@@ -119,13 +125,13 @@ __global__ void __launch_bounds__(256)
       }
     }
 #pragma unroll
-    for (int n = 0; n < 8; ++n)
+    for (int n = 0; n < NS; ++n)
 #pragma unroll
       for (int e = 0; e < 4; ++e)
         if (n * 8 + (lane & 3) * 2 + (e & 1) >= nvalid) s[n][e] = -INFINITY;
     float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
+    for (int n = 0; n < NS; ++n) {
       mx0 = fmaxf(mx0, fmaxf(s[n][0], s[n][1]));
       mx1 = fmaxf(mx1, fmaxf(s[n][2], s[n][3]));
     }
@@ -140,7 +146,7 @@ __global__ void __launch_bounds__(256)
     rmax[1] = n1;
     float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
+    for (int n = 0; n < NS; ++n) {
       s[n][0] = exp2f((s[n][0] - b0) * sl2);
       s[n][1] = exp2f((s[n][1] - b0) * sl2);
       s[n][2] = exp2f((s[n][2] - b1) * sl2);
@@ -155,9 +161,9 @@ __global__ void __launch_bounds__(256)
       o[n][0] *= sc0; o[n][1] *= sc0;
       o[n][2] *= sc1; o[n][3] *= sc1;
     }
-    // P V over the 64 rows in four 16-row steps; P = hi + lo, both bf16
+    // P V over the CH rows in 16-row steps; P = hi + lo, both bf16
 #pragma unroll
-    for (int ks = 0; ks < 4; ++ks) {
+    for (int ks = 0; ks < CH / 16; ++ks) {
       uint32_t ph[4], pl[4];
       const float* q0 = s[2 * ks];
       const float* q1 = s[2 * ks + 1];
@@ -287,18 +293,25 @@ int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s) {
   int seg_rows = (p.rows + kPrefillMaxSeg - 1) / kPrefillMaxSeg;
   seg_rows = std::max(kPfChunk, (seg_rows + kPfChunk - 1) / kPfChunk * kPfChunk);
   const int nseg = (p.rows + seg_rows - 1) / seg_rows;
-  const size_t smem = ((size_t)rep * 16 + 4 * kPfChunk) * kPfLd * sizeof(bf16);
+  // K/V rows per pipeline stage (LSP_PREFILL_CHUNK=16|32|64 overrides, for measurement)
+  int ch = kPrefillStage;
+  if (const char* v = std::getenv("LSP_PREFILL_CHUNK")) {
+    const int w = std::atoi(v);
+    ch = w == 16 ? 16 : (w == 64 ? 64 : 32);
+  }
+  const size_t smem = ((size_t)rep * 16 + 4 * ch) * kPfLd * sizeof(bf16);
   if (smem > 227 * 1024) return LSP_ERR_SHAPE;
-  static size_t attr = 0;
+  auto kern = ch == 16 ? prefill_partial_kernel<16> : ch == 32 ? prefill_partial_kernel<32> : prefill_partial_kernel<64>;
+  static size_t attr_by[3] = {0, 0, 0};
+  size_t& attr = attr_by[ch == 16 ? 0 : ch == 32 ? 1 : 2];
   if (smem > attr) {
-    if (cudaFuncSetAttribute(prefill_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return LSP_ERR_CUDA;
     attr = smem;
   }
   // R = 0 (no summary): only the window, boundary and t are written
-  if ((p.R > 0 && launch_pdl(prefill_partial_kernel, dim3(nseg, p.L * p.nkv), dim3(rep * 32), smem, s, p,
-                             rep, seg_rows) != cudaSuccess) ||
+  if ((p.R > 0 && launch_pdl(kern, dim3(nseg, p.L * p.nkv), dim3(rep * 32), smem, s, p, rep, seg_rows) !=
+                      cudaSuccess) ||
       launch_pdl(prefill_merge_kernel<bf16>, dim3(p.L * p.nq + p.L * p.nkv), dim3(256), 0, s, p, nseg) !=
           cudaSuccess)
     return LSP_ERR_CUDA;
