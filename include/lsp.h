@@ -303,7 +303,13 @@ int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_log
  *   LSP_GEMM_CLUSTER=1 and splits 2, 4 or 8 instead, the split CTAs of each
  *   128-row weight tile form a thread-block cluster that sums its partials in
  *   distributed shared memory, in split order, and writes Y (workspace unused;
- *   the drafter's projections then reduce the same way). */
+ *   the drafter's projections then reduce the same way).
+ *   Two more variables change how the work is laid out, never the result:
+ *   LSP_GEMM_TOKG=G (2..4) splits the M tokens over G CTAs per weight tile
+ *   (LSP_GEMM_TOKG_GU for the drafter's SwiGLU gate/up projection alone,
+ *   which takes 2 by default at M >= 128 when its tiles fill less than one
+ *   wave), and LSP_GEMM_MCAST=1 pairs CTAs of adjacent weight tiles in
+ *   clusters that share each activation tile by TMA multicast. */
 size_t lsp_linear_workspace_bytes(int M, int N, int splits);
 int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype,
                int splits, void* workspace, size_t workspace_bytes, lsp_stream_t stream);

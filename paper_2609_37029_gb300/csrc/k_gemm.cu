@@ -107,12 +107,14 @@ constexpr uint32_t kXchgBytes = 17408;                        // 128 x 33 floats
 // loads its row's TT accumulators, writes them (or, for SwiGLU, the
 // activation of its share after a gate/up exchange) into staging buffer
 // c & 1, and one thread stores the buffer with a TMA tensor store into the
-// [split][token][feature] view of Y.  Token rows past M and feature columns
-// past N fall outside the view and are not written.
+// [split][token][feature] view of Y at the CTA's first token row tok0.
+// Token rows past M and feature columns past N fall outside the view and are
+// not written; the chunks tile the CTA's m_pad tokens exactly, so no store
+// reaches the next token group's rows.
 template <typename T>
 __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensorMap* to, uint8_t* smem,
-                                             uint32_t lane_base, int ntl, int tile0, int split,
-                                             int r) {
+                                             uint32_t lane_base, int ntl, int tile0, int tok0,
+                                             int split, int r) {
   const bool swiglu = p.mode == EPI_SWIGLU;
   const bool f32out = p.mode == EPI_F32 || p.mode == EPI_PARTIAL;
   const int es = f32out ? 4 : (int)sizeof(T);
@@ -122,9 +124,10 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
   uint8_t* stg0 = smem + (swiglu ? kXchgBytes : 0);
   const uint32_t buf_bytes = (uint32_t)(TT * cols * es);     // <= 16 KB
   const bool issuer = r == 0;
+  const int m_end = min(p.m_pad, p.M - tok0);                 // > 0: no token group is empty
   int chunk = 0;
   for (int w = 0; w < ntl; ++w) {
-    for (int m0 = 0; m0 < p.m_pad; m0 += TT, ++chunk) {
+    for (int m0 = 0; m0 < m_end; m0 += TT, ++chunk) {       // no store box starts past row M
       float v[32];
       const uint32_t col = (uint32_t)(w * p.m_pad + m0);
       if (TT == 32) tmem_ld32(lane_base + col, v);
@@ -162,7 +165,7 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
       fence_proxy_async_smem();
       named_bar(1, kEpilogueThreads);
       if (issuer) {
-        tma_store_3d(to, smem_u32(stg), (tile0 + w) * cols, m0, split);
+        tma_store_3d(to, smem_u32(stg), (tile0 + w) * cols, tok0 + m0, split);
         bulk_commit();
       }
     }
@@ -252,8 +255,8 @@ __device__ __forceinline__ void epilogue_cluster(const GemmParams& p, uint8_t* s
   }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+template <typename T, int kOcc>
+__global__ void __launch_bounds__(kGemmThreads, kOcc)
     gemm_kernel(const __grid_constant__ CUtensorMap ta0, const __grid_constant__ CUtensorMap ta1,
                 const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb,
                 const __grid_constant__ CUtensorMap to, const __grid_constant__ GemmParams p) {
@@ -270,7 +273,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int tile0 = blockIdx.x * p.wt;
+  // blockIdx.x = weight-tile CTA x token groups + group: the CTAs of one weight
+  // tile are adjacent, so they run together and share the tile through L2
+  const int group = (int)blockIdx.x % p.tok_groups;
+  const int tile0 = ((int)blockIdx.x / p.tok_groups) * p.wt;
+  const int tok0 = group * p.m_pad;                            // first token row of this CTA
   const int ntl = min(p.wt, p.n_tiles - tile0);                // weight tiles of this CTA
   const int split = blockIdx.y;
   const int kb0 = (int)((long long)split * p.kblocks / p.splits);
@@ -283,10 +290,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
   const uint32_t acc_bar = bar0 + 8u * (2 * S);
 
+  // Activation multicast (p.mcast): the two CTAs of a cluster hold adjacent
+  // weight tiles and the same tokens; each loads half of every activation box
+  // into both, and a stage is refilled only after both released it.
+  const bool mcast = p.mcast != 0;
+  const uint32_t crank = mcast ? cluster_ctarank() : 0u;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+      mbar_init(empty_bar(s), mcast ? 2 : 1);
     }
     mbar_init(acc_bar, 1);
     *s_abort = 0;
@@ -298,6 +310,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), (uint32_t)p.tmem_cols);
   tc_fence_before();
   __syncthreads();
+  if (mcast) cluster_sync_all();          // the peer's barriers exist before anything lands in them
   tc_fence_after();
   griddep_launch();
   const uint32_t tmem_base = *tmem_slot;
@@ -305,7 +318,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   int issued = 0;
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA producer
-    const uint64_t pol_w = policy_evict_first();
+    // a weight tile read by one CTA goes first; shared by token groups, it stays
+    const uint64_t pol_w = p.tok_groups > 1 ? policy_evict_normal() : policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
     // weight tile w of this CTA: segment (tensor map) and first row within it
     auto a_seg = [&](int w) {
@@ -328,6 +342,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     };
     auto prefetch_a = [&](int i) {
+      if (group != 0) return;                // one CTA of the tile prefetches it
       const int kx = (kb0 + i) * G::BK;
       for (int w = 0; w < ntl; ++w) {
         if (p.mode == EPI_SWIGLU) {
@@ -341,8 +356,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     };
     auto load_b = [&](int i, uint32_t sb, uint32_t bar) {
       const int kx = (kb0 + i) * G::BK;
-      for (int tt = 0; tt < p.n_tok_tiles; ++tt)
-        tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, bar, kx, tt * p.bn, pol_x);
+      for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
+        if (mcast) {                          // rows [crank * bn/2, +bn/2) of the box, to both CTAs
+          const int h = p.bn / 2, r0 = tt * p.bn + (int)crank * h;
+          tma_load_2d_mc(sb + (uint32_t)(r0 * 128), &tb, bar, kx, tok0 + r0, (uint16_t)0x3, pol_x);
+        } else {
+          tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, bar, kx, tok0 + tt * p.bn, pol_x);
+        }
+      }
     };
     // Weights do not depend on the preceding kernel: start streaming them now.
     int next_pf = 0;
@@ -392,7 +413,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
         }
       }
-      umma_commit(empty_bar(s));
+      if (mcast) umma_commit_mc(empty_bar(s), (uint16_t)0x3);
+      else umma_commit(empty_bar(s));
     }
     umma_commit(acc_bar);
   } else if (warp >= 2) {
@@ -409,14 +431,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (p.creduce) {
       // reduced across the cluster below, by the whole CTA
     } else if (*s_abort == 0 && p.tma_out) {
-      epilogue_tma<T>(p, &to, smem, lane_base, ntl, tile0, split, r);
+      epilogue_tma<T>(p, &to, smem, lane_base, ntl, tile0, tok0, split, r);
     } else if (*s_abort == 0) {
       for (int w = 0; w < ntl; ++w)
         for (int tt = 0; tt < p.n_tok_tiles; ++tt)
           for (int c0 = 0; c0 < p.bn; c0 += 16) {
             float v[16];
             tmem_ld16(lane_base + (uint32_t)((w * p.n_tok_tiles + tt) * p.bn + c0), v);
-            emit_chunk<T>(p, tile0 + w, split, r, tt * p.bn + c0, v, xchg);
+            emit_chunk<T>(p, tile0 + w, split, r, tok0 + tt * p.bn + c0, v, xchg);
           }
     }
   }
@@ -427,6 +449,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // A wait gave up: let every TMA copy this CTA issued land before exit.
     for (int i = (issued > S ? issued - S : 0); i < issued; ++i)
       mbar_wait(full_bar(i % S), (uint32_t)(i / S) & 1u, p.err);
+  }
+  if (mcast) {
+    // The peer's last releases arrive on this CTA's barriers: take them all
+    // before either CTA of the pair exits.
+    if (warp == 0 && lane == 0 && *s_abort == 0)
+      for (int i = (nk > S ? nk - S : 0); i < nk; ++i)
+        if (!mbar_wait(empty_bar(i % S), (uint32_t)(i / S) & 1u, p.err)) break;
+    __syncwarp();
+    cluster_sync_all();
   }
   if (p.creduce) {
     // the stage ring is idle: every load landed before the last MMA was issued
@@ -529,8 +560,10 @@ static void token_tiling(int M, int* bn, int* ntt) {
 static constexpr int kSmemBudget = 227 * 1024;
 
 // Tuning overrides for measurement sweeps: LSP_GEMM_WT (weight tiles per CTA),
-// LSP_GEMM_PD (L2 prefetch distance in k-blocks), LSP_GEMM_STAGES.  Unset or
-// non-positive values keep the defaults; the values never change results.
+// LSP_GEMM_PD (L2 prefetch distance in k-blocks), LSP_GEMM_STAGES,
+// LSP_GEMM_TOKG (token groups; LSP_GEMM_TOKG_GU for the SwiGLU gate/up
+// projection alone).  Unset or non-positive values keep the defaults; the
+// values never change results.
 static int tuning(const char* name) {
   const char* v = std::getenv(name);
   return v ? std::atoi(v) : 0;
@@ -548,6 +581,45 @@ static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
   return ctas * 4 >= (long long)num_sms * 5 && two_per_sm_fits(wt, m_pad);
 }
 
+// Three 2-stage CTAs per SM (shared memory incl. the 1 KB each CTA reserves,
+// TMEM columns, and the kernel instance bounded to 3 x 192 threads' registers)
+// when there are enough CTAs to give most SMs a third.  Used with token groups
+// (or, for sweeps, LSP_GEMM_OCC3=1).
+constexpr int kSmemPerSm = 228 * 1024;
+static bool three_per_sm_fits(int wt, int m_pad, int groups) {
+  if (groups < 2 && tuning("LSP_GEMM_OCC3") <= 0) return false;
+  int cols = 32;
+  while (cols < wt * m_pad) cols *= 2;
+  const int stage_bytes = wt * (int)kTileBytes + m_pad * 128;
+  return 3 * (2 * stage_bytes + 1280 + 1024) <= kSmemPerSm && 3 * cols <= 512;
+}
+
+static bool use_three_per_sm(long long ctas, int num_sms, int wt, int m_pad, int groups) {
+  return ctas >= 2LL * num_sms && three_per_sm_fits(wt, m_pad, groups);
+}
+
+// Token groups: the CTAs of a weight tile split the M tokens G ways (each
+// streams the tile; the copies after the first come from L2).  Smaller stages
+// let three CTAs share an SM.  Default: two groups for the SwiGLU gate/up
+// projection when its tiles fill less than one wave of two CTAs per SM and two
+// groups reach three per SM (Qwen3-8B round, M = 256, 192 tiles: gate/up 368 ->
+// 359 us per round, round 1.243 -> 1.231 ms); one otherwise (the other
+// projections and the LM head measured slower with two: more CTAs re-stream
+// each weight tile for the same work).
+static int token_groups(int M, int mode, int n_tiles, int num_sms) {
+  int req = mode == EPI_SWIGLU && M >= 128 && n_tiles <= 2 * num_sms && n_tiles >= num_sms ? 2 : 1;
+  if (tuning("LSP_GEMM_TOKG") > 0) req = tuning("LSP_GEMM_TOKG");
+  if (mode == EPI_SWIGLU && tuning("LSP_GEMM_TOKG_GU") > 0) req = tuning("LSP_GEMM_TOKG_GU");
+  int g = std::min(std::min(std::max(1, req), 4), std::max(1, M / 16));
+  // every group holds at least one token row
+  for (; g > 1; --g) {
+    int bn, ntt;
+    token_tiling((M + g - 1) / g, &bn, &ntt);
+    if ((g - 1) * bn * ntt < M) break;
+  }
+  return g;
+}
+
 // Split-K factor from a cost model in units of one k-block of one of two
 // co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
 // fixed per-CTA cost) + the cost of combining the splits (fixed_cost +
@@ -557,16 +629,17 @@ static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
 // lone CTA is no faster: its single MMA issuer keeps the tensor pipe only
 // partly busy, and a second CTA on the SM hides that.
 int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
-                     int max_splits, bool two_ok, bool wide) {
+                     int max_splits, int occ_max, bool wide) {
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(max_splits, kblocks); ++s) {
     if (max_splits == kMaxClusterSplits && s > 1 && (s & (s - 1))) continue;   // cluster sizes 2, 4, 8
     const long long ctas = (long long)n_ctas * s;
-    const bool two = two_ok && ctas * 4 >= (long long)num_sms * 5;
-    const long long slots = two ? 2LL * num_sms : num_sms;
+    const int occ = (occ_max >= 3 && ctas >= 2LL * num_sms) ? 3
+                    : (occ_max >= 2 && ctas * 4 >= (long long)num_sms * 5) ? 2 : 1;
+    const long long slots = (long long)occ * num_sms;
     const long long waves = (ctas + slots - 1) / slots;
-    const double per = (double)((kblocks + s - 1) / s) * (two || wide ? 1.0 : 0.63) + 2.0;
+    const double per = (double)((kblocks + s - 1) / s) * (occ > 1 || wide ? 1.0 : 0.63) + 2.0;
     const double cost = (double)waves * per + (s > 1 ? fixed_cost + per_split_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
@@ -588,25 +661,39 @@ bool gemm_cluster_enabled() {
   return v && v[0] == '1';
 }
 
+// Activation multicast across CTA pairs, opt-in (LSP_GEMM_MCAST=1).  Measured
+// at the Qwen3-8B drafting round it is slightly slower (LM head 267 vs 261 us,
+// round 1.269 vs 1.242 ms): halving the activation tile's L2 reads does not
+// shorten the weight stream, so each CTA loads its whole activation tile.
+bool gemm_mcast_enabled() {
+  const char* v = std::getenv("LSP_GEMM_MCAST");
+  return v && v[0] == '1';
+}
+
 // Model cost of one in-cluster reduction, k-block units: two cluster barriers
 // per pass and the distributed-shared-memory reads of the peers' dumps.
 constexpr double kClusterReduceCost = 1.5;
 
-void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt) {
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt,
+                 int* groups) {
+  const int G = token_groups(M, mode, n_tiles, num_sms);
+  if (groups) *groups = G;
   int bn, ntt;
-  token_tiling(M, &bn, &ntt);
+  token_tiling((M + G - 1) / G, &bn, &ntt);
   const int m_pad = bn * ntt;
   // one weight tile per CTA: two tiles sharing the activation tile measured slower
   if (*wt <= 0) *wt = 1;
   const int kblocks = gemm_kblocks(K, dtype);
-  const int n_ctas = (n_tiles + *wt - 1) / *wt;
-  const bool two = two_per_sm_fits(*wt, m_pad), wide = m_pad >= 128;
+  const int n_ctas = (n_tiles + *wt - 1) / *wt * G;
+  const int occ_max = three_per_sm_fits(*wt, m_pad, G) ? 3 : two_per_sm_fits(*wt, m_pad) ? 2 : 1;
+  const bool wide = m_pad >= 128;
   if (*splits <= 0) {
-    if (gemm_cluster_enabled() && *wt == 1)
-      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, 0.0, kClusterReduceCost, kMaxClusterSplits, two, wide);
+    if (gemm_cluster_enabled() && *wt == 1 && G == 1)
+      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, 0.0, kClusterReduceCost, kMaxClusterSplits,
+                                 std::min(occ_max, 2), wide);
     else if (mode == EPI_PARTIAL)
       *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows), 0.0, 16,
-                                 two, wide);
+                                 occ_max, wide);
     else
       *splits = 1;
   }
@@ -641,10 +728,12 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     for (int i = 0; i < nseg; ++i) p.N += seg_rows[i];
   }
   p.kblocks = gemm_kblocks(K, dtype);
-  token_tiling(M, &p.bn, &p.n_tok_tiles);
-  p.m_pad = p.bn * p.n_tok_tiles;
   if (wt <= 0 && tuning("LSP_GEMM_WT") > 0) wt = tuning("LSP_GEMM_WT");
-  gemm_choose(dtype, M, K, p.n_tiles, mode, num_sms, &splits, &wt);
+  int G = 1;
+  gemm_choose(dtype, M, K, p.n_tiles, mode, num_sms, &splits, &wt, &G);
+  p.tok_groups = G;
+  token_tiling((M + G - 1) / G, &p.bn, &p.n_tok_tiles);      // per token group
+  p.m_pad = p.bn * p.n_tok_tiles;
   if (wt < 1 || wt > 2 || wt * p.m_pad > 512) return LSP_ERR_SHAPE;
   p.wt = wt;
   int cols = 32;
@@ -652,8 +741,14 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   p.tmem_cols = cols;
   const int stage_bytes = wt * (int)kTileBytes + p.m_pad * 128;
   p.stages = std::min(8, (kSmemBudget - 2048) / stage_bytes);
-  const int n_ctas = (p.n_tiles + wt - 1) / wt;
-  if (use_two_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad)) p.stages = 2;
+  const int n_ctas = (p.n_tiles + wt - 1) / wt * G;
+  op->occ = 1;
+  if (use_three_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad, G)) {
+    p.stages = 2;
+    op->occ = 3;
+  } else if (use_two_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad)) {
+    p.stages = 2;
+  }
   if (tuning("LSP_GEMM_STAGES") > 0) p.stages = std::min(p.stages, tuning("LSP_GEMM_STAGES"));
   if (p.stages < 2) return LSP_ERR_SHAPE;
   // L2 prefetch of each weight tile issued before waiting for its smem slot
@@ -663,9 +758,12 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
   p.splits = splits;
   // split-K: reduced in a cluster of the tile's split CTAs when possible
   // (power-of-two clusters: a cluster of 6 measured 23 co-resident clusters, not 48)
-  p.creduce = (splits == 2 || splits == 4 || splits == 8) && wt == 1 && gemm_cluster_enabled() ? 1 : 0;
+  p.creduce = (splits == 2 || splits == 4 || splits == 8) && wt == 1 && G == 1 && gemm_cluster_enabled() ? 1 : 0;
   if (splits > 1 && mode != EPI_PARTIAL && !p.creduce) return LSP_ERR_SHAPE;
   p.out_splits = p.creduce ? 1 : splits;
+  // each CTA of a pair loads bn/2 rows of every activation box (a whole number
+  // of 8-row swizzle atoms: bn is a multiple of 16)
+  p.mcast = wt == 1 && G == 1 && !p.creduce && p.n_tiles >= 2 && gemm_mcast_enabled() ? 1 : 0;
   // tokens per reduction pass: the stage ring holds a [tokens][128] fp32 dump
   p.cr_tok = std::min(p.m_pad, (int)((size_t)p.stages * stage_bytes / (kTileRows * 4) / 16 * 16));
   if (p.creduce && p.cr_tok < 16) return LSP_ERR_SHAPE;
@@ -679,7 +777,7 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     const int si = i < nseg ? i : 0;
     if ((rc = make_map(&op->a[i], dtype, W[si], K, seg_rows[si], box_rows)) != LSP_OK) return rc;
   }
-  if ((rc = make_map(&op->b, dtype, X, K, M, p.bn)) != LSP_OK) return rc;
+  if ((rc = make_map(&op->b, dtype, X, K, M, p.mcast ? p.bn / 2 : p.bn)) != LSP_OK) return rc;
   // TMA-store epilogue when the output view can be described (else per-thread stores)
   p.out_tok = (p.m_pad % 32) ? 16 : 32;
   {
@@ -689,24 +787,27 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
                 std::getenv("LSP_GEMM_SCALAR_EPI") == nullptr;
     if (!p.tma_out) op->out = op->b;       // unused placeholder
   }
-  op->grid = dim3((unsigned)n_ctas, (unsigned)splits, 1);
+  op->grid = dim3((unsigned)(p.mcast ? (n_ctas + 1) / 2 * 2 : n_ctas), (unsigned)splits, 1);
   op->cluster = p.creduce ? splits : 1;
   op->smem = (size_t)p.stages * stage_bytes + 1024 + 256;
   return LSP_OK;
 }
 
-template <typename T>
+template <typename T, int kOcc>
 static int launch_t(const GemmOp* op, cudaStream_t s) {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(gemm_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+    cudaFuncSetAttribute(gemm_kernel<T, kOcc>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+    if (kOcc > 1)   // room for kOcc CTAs' shared memory on one SM
+      cudaFuncSetAttribute(gemm_kernel<T, kOcc>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   });
-  if (op->cluster <= 1) {
-    const cudaError_t e = launch_pdl(gemm_kernel<T>, op->grid, dim3(kGemmThreads), op->smem, s,
+  if (op->cluster <= 1 && !op->p.mcast) {
+    const cudaError_t e = launch_pdl(gemm_kernel<T, kOcc>, op->grid, dim3(kGemmThreads), op->smem, s,
                                      op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
     return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
   }
-  // the split CTAs of a weight tile form one cluster (grid.y == cluster size)
+  // the split CTAs of a weight tile form one cluster (grid.y == cluster size),
+  // or two adjacent weight tiles do (activation multicast)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = op->grid;
   cfg.blockDim = dim3(kGemmThreads);
@@ -716,18 +817,19 @@ static int launch_t(const GemmOp* op, cudaStream_t s) {
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = 1;
-  attr[1].val.clusterDim.y = (unsigned)op->cluster;
+  attr[1].val.clusterDim.x = op->p.mcast ? 2u : 1u;
+  attr[1].val.clusterDim.y = op->p.mcast ? 1u : (unsigned)op->cluster;
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_kernel<T>, op->a[0], op->a[1], op->a[2], op->b,
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_kernel<T, kOcc>, op->a[0], op->a[1], op->a[2], op->b,
                                            op->out, op->p);
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 int gemm_launch(const GemmOp* op, cudaStream_t s) {
-  return op->dtype == LSP_DTYPE_BF16 ? launch_t<bf16>(op, s) : launch_t<float>(op, s);
+  if (op->occ == 3) return op->dtype == LSP_DTYPE_BF16 ? launch_t<bf16, 3>(op, s) : launch_t<float, 3>(op, s);
+  return op->dtype == LSP_DTYPE_BF16 ? launch_t<bf16, 1>(op, s) : launch_t<float, 1>(op, s);
 }
 
 int launch_sum_partials(const float* part, int splits, size_t n, float* y, cudaStream_t s) {

@@ -55,6 +55,9 @@ struct GemmParams {
                         //    distributed shared memory; the output is final (one slice)
   int cr_tok;           // tokens per cluster-reduction pass (the idle stage ring holds them)
   int out_splits;       // slices of the output the consumer sums (splits, or 1 when reduced)
+  int tok_groups;       // CTAs per weight tile, each over m_pad consecutive tokens
+  int mcast;            // 1: CTA pairs (clusters of 2 along x) share each activation box by TMA
+                        //    multicast; grid.x is even (a CTA past the last tile only loads)
   void* Y;
   int ldy;
   unsigned* err;
@@ -68,6 +71,7 @@ struct GemmOp {
   int dtype;
   dim3 grid;
   int cluster;          // CTAs per cluster along the split axis (1: no cluster)
+  int occ;              // CTAs per SM the plan sizes for: 3 picks the register-bounded instance
   size_t smem;
 };
 
@@ -83,13 +87,17 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
               const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
               int num_sms, int splits, int wt);
 int gemm_launch(const GemmOp* op, cudaStream_t s);
-// The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 = choose).
-void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt);
+// The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 =
+// choose), and the token groups it splits M into (groups may be null).
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt,
+                 int* groups = nullptr);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
+// occ_max: CTAs one SM can hold (1-3) for this tile shape.
 int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
-                     int max_splits, bool two_ok, bool wide);
+                     int max_splits, int occ_max, bool wide);
 constexpr int kMaxClusterSplits = 8;    // portable cluster size
 bool gemm_cluster_enabled();
+bool gemm_mcast_enabled();
 double gemm_partial_cost(int M, int N);
 int gemm_kblocks(int K, int dtype);
 // Deterministic sum of `splits` fp32 partials [splits][n] into y[n].
