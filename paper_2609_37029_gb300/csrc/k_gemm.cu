@@ -646,12 +646,21 @@ static int token_groups(int M, int mode, int n_tiles, int num_sms) {
 // co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
 // fixed per-CTA cost) + the cost of combining the splits (fixed_cost +
 // per_split_cost per split: the consumer's re-read of fp32 partials from L2,
-// or the in-cluster reduction).  With a small token tile a lone CTA on an SM
-// streams a k-block in ~0.63 of that time; with a wide one (>= 128 tokens) a
-// lone CTA is no faster: its single MMA issuer keeps the tensor pipe only
-// partly busy, and a second CTA on the SM hides that.
+// or the in-cluster reduction).  A lone CTA on an SM, with its deeper ring,
+// moves a k-block in 0.53 of that time (0.42 vs 0.80 us measured at M = 256
+// with the MMA issue loop at 0.24 us per k-block; LSP_GEMM_LONE_COST
+// overrides the factor for sweeps, and a negative value restores the fit made
+// before that loop was trimmed: 0.63 below 128 tokens, 1.0 from 128).
+static double lone_cta_cost(bool wide) {
+  const char* v = std::getenv("LSP_GEMM_LONE_COST");
+  const double f = v ? std::atof(v) : 0.53;
+  if (f < 0) return wide ? 1.0 : 0.63;
+  return f > 0 ? f : 0.53;
+}
+
 int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
                      int max_splits, int occ_max, bool wide) {
+  const double lone = lone_cta_cost(wide);
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(max_splits, kblocks); ++s) {
@@ -661,7 +670,7 @@ int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost
                     : (occ_max >= 2 && ctas * 4 >= (long long)num_sms * 5) ? 2 : 1;
     const long long slots = (long long)occ * num_sms;
     const long long waves = (ctas + slots - 1) / slots;
-    const double per = (double)((kblocks + s - 1) / s) * (occ > 1 || wide ? 1.0 : 0.63) + 2.0;
+    const double per = (double)((kblocks + s - 1) / s) * (occ > 1 ? 1.0 : lone) + 2.0;
     const double cost = (double)waves * per + (s > 1 ? fixed_cost + per_split_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
