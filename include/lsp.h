@@ -311,6 +311,20 @@ int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_log
  *   wave), and LSP_GEMM_MCAST=1 pairs CTAs of adjacent weight tiles in
  *   clusters that share each activation tile by TMA multicast. */
 size_t lsp_linear_workspace_bytes(int M, int N, int splits);
+
+/* Diagnostic, host only (needs no GPU): the launch plan the drafter's
+ * projection GEMM takes for M token rows, N output features and reduction
+ * length K on a device with num_sms SMs, under the current environment
+ * (the LSP_GEMM_* variables above).
+ *   swiglu = 0: a projection whose fp32 split-K partials a consumer sums
+ *   (the q/k/v, o, down and boundary-fusion projections); swiglu = 1: the
+ *   fused gate/up projection with N = F (gate and up each [F][K]).
+ *   *splits: split-K factor; *tok_groups: CTAs per weight tile, each over
+ *   *tokens_per_group consecutive token rows (a multiple of 16).
+ * LSP_ERR_ARG for null outputs, M outside [1, 512], N, K or num_sms < 1 or
+ * an unknown dtype. */
+int lsp_gemm_plan_info(int dtype, int M, int N, int K, int swiglu, int num_sms, int* splits,
+                       int* tok_groups, int* tokens_per_group);
 int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int dtype,
                int splits, void* workspace, size_t workspace_bytes, lsp_stream_t stream);
 

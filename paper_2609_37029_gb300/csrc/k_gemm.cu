@@ -579,6 +579,12 @@ static void token_tiling(int M, int* bn, int* ntt) {
   *bn = std::max(16, (per + 15) / 16 * 16);
 }
 
+int gemm_group_rows(int M, int G) {
+  int bn, ntt;
+  token_tiling((M + G - 1) / G, &bn, &ntt);
+  return bn * ntt;
+}
+
 static constexpr int kSmemBudget = 227 * 1024;
 
 // Tuning overrides for measurement sweeps: LSP_GEMM_WT (weight tiles per CTA),

@@ -533,6 +533,21 @@ int lsp_sample(lsp_state* st, const float* base_logits, const int32_t* prev_toke
   return run_sampler(st, base_logits, out_logits, prev_token, 1, Ec, Wc, sp, out_tokens, S(stream));
 }
 
+int lsp_gemm_plan_info(int dtype, int M, int N, int K, int swiglu, int num_sms, int* splits,
+                       int* tok_groups, int* tokens_per_group) {
+  if (!splits || !tok_groups || !tokens_per_group || M < 1 || M > 512 || N < 1 || K < 1 || num_sms < 1)
+    return LSP_ERR_ARG;
+  if (dtype != LSP_DTYPE_BF16 && dtype != LSP_DTYPE_F32) return LSP_ERR_ARG;
+  const int mode = swiglu ? EPI_SWIGLU : EPI_PARTIAL;
+  const int rows[1] = {N};
+  int s = 0, wt = 0, g = 1;
+  gemm_choose(dtype, M, K, gemm_tiles(mode, rows, 1), mode, num_sms, &s, &wt, &g);
+  *splits = s;
+  *tok_groups = g;
+  *tokens_per_group = gemm_group_rows(M, g);
+  return LSP_OK;
+}
+
 size_t lsp_linear_workspace_bytes(int M, int N, int splits) {
   if (M < 1 || N < 1 || splits < 1) return 0;
   return splits == 1 ? 0 : (size_t)splits * M * N * sizeof(float);

@@ -92,6 +92,8 @@ int gemm_launch(const GemmOp* op, cudaStream_t s);
 void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt,
                  int* groups = nullptr);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
+// Token rows one token group of M rows split G ways covers (a multiple of 16).
+int gemm_group_rows(int M, int G);
 // occ_max: CTAs one SM can hold (1-3) for this tile shape.
 int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
                      int max_splits, int occ_max, bool wide);

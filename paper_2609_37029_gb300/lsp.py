@@ -90,6 +90,8 @@ _f = {
                                c_int, c_int, c_int, c_int, c_int, POINTER(lsp_sample_params),
                                c_void_p, c_void_p, c_void_p, c_void_p),
     "lsp_linear_workspace_bytes": _sig("lsp_linear_workspace_bytes", c_size_t, c_int, c_int, c_int),
+    "lsp_gemm_plan_info": _sig("lsp_gemm_plan_info", c_int, c_int, c_int, c_int, c_int, c_int, c_int,
+                               POINTER(c_int), POINTER(c_int), POINTER(c_int)),
     "lsp_linear": _sig("lsp_linear", c_int, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                        c_int, c_void_p, c_size_t, c_void_p),
     "lsp_philox_words": _sig("lsp_philox_words", c_int, c_uint64, c_uint32, c_uint32, c_uint32,
@@ -226,6 +228,14 @@ def lsp_sample_noalloc(base_logits, prev_token, Ec, Wc, dtype, C, B, V, rc,
 
 def lsp_linear_workspace_bytes(M: int, N: int, splits: int) -> int:
     return _f["lsp_linear_workspace_bytes"](M, N, splits)
+
+
+def lsp_gemm_plan_info(dtype, M, N, K, swiglu, num_sms):
+    """(splits, token groups, token rows per group) of the projection GEMM's plan (host only)."""
+    s, g, r = c_int(0), c_int(0), c_int(0)
+    _check(_f["lsp_gemm_plan_info"](dtype, M, N, K, int(bool(swiglu)), num_sms, ctypes.byref(s),
+                                    ctypes.byref(g), ctypes.byref(r)), "lsp_gemm_plan_info")
+    return s.value, g.value, r.value
 
 
 def lsp_linear(X, W, Y, M, N, K, dtype, splits=1, workspace=None, workspace_bytes=0,
