@@ -6,15 +6,23 @@
 // large weight.  The kernel therefore puts 128 weight rows on the UMMA M axis
 // and the tokens on its N axis ("swap AB"): D^T[n][m] = sum_k W[n][k] X[m][k].
 //
-//   warp 0      TMA producer: `wt` 128 x BK weight tiles and the M x BK
-//               activation tile per stage into an S-deep mbarrier ring, plus
-//               L2 prefetches of the weight tiles `pd` stages ahead
-//   warp 1      TMEM allocation and the single-thread tcgen05.mma issue
+//   warp 0      TMA producer: `wt` 128 x BK weight tiles and the CTA's
+//               m_pad x BK activation tile per stage into an S-deep mbarrier
+//               ring, plus L2 prefetches of the weight tiles `pd` stages ahead
+//   warp 1      TMEM allocation and the single-thread tcgen05.mma issue (a
+//               lean loop: this one thread's instructions set the issue rate)
 //   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulators, the fused
 //               output (fp32, storage dtype, SwiGLU, or a split-K partial)
 //               staged in shared memory 16-32 tokens at a time and written
 //               by TMA tensor stores (double-buffered), so the global writes
 //               are full-line bulk copies that overlap the next chunk
+//
+// Grid: x = weight-tile CTAs x token groups (a group's CTAs share the weight
+// tile, each over m_pad consecutive tokens; the SwiGLU gate/up projection
+// takes two groups when its tiles fill under one wave of two CTAs per SM),
+// y = split-K.  Kept opt-in after measuring slower: split-K reduced inside a
+// cluster (LSP_GEMM_CLUSTER=1) and activation multicast across CTA pairs
+// (LSP_GEMM_MCAST=1).
 //
 // Launched as a programmatic dependent: before the preceding kernel finishes,
 // the producer already streams this launch's weights (L2 prefetch and the
