@@ -96,3 +96,25 @@ def test_verification_randomness_is_a_separate_philox_stream():
     assert not np.array_equal(d, a) and not np.array_equal(d, g) and not np.array_equal(a, g)
     u = verify.accept_uniform(5, 1, 0, 0)
     assert 0.0 < u < 1.0 and u == (float(a[0] >> np.uint32(9)) + 0.5) * 2.0 ** -23
+
+
+def test_accepted_length_is_truncated_geometric_in_alpha():
+    """With the same (p, q) at every position, each candidate is accepted with probability
+    alpha = sum_v min(p(v), q(v)) independently of the others, and the round stops at the
+    first rejection: P(r = k) = alpha^k (1 - alpha) for k < B and P(r = B) = alpha^B.
+    Accepting past a rejection, or a per-position ratio other than p/q, breaks it."""
+    B, n, T = 3, 6000, 1.0
+    zq1 = ZQ[0]
+    zt = np.stack([ZT[0]] * (B + 1))
+    zq = np.stack([zq1] * B)
+    hist = np.zeros(B + 1)
+    for k in range(n):
+        seed = 7000 + k
+        y = [int(np.argmax(zq[i] / T + gumbel(seed, 5, 2, i, V))) for i in range(B)]
+        r, _, _, _ = verify.verify_block(zt, zq, y, T, seed, 5, 2)
+        hist[r] += 1
+    a = np.minimum(_softmax(ZT[0] / T), _softmax(zq1 / T)).sum()
+    want = np.array([a ** j * (1 - a) for j in range(B)] + [a ** B])
+    got = hist / n
+    assert np.all(np.abs(got - want) <= 5 * np.sqrt(want * (1 - want) / n) + 1e-3), (got, want)
+    assert 0.2 < a < 0.8                     # every length has weight: the law is visible
