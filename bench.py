@@ -331,40 +331,61 @@ def variants_leg(s, lsp, seed_base, dist, steps=100, prefix=4096):
 
 # ------------------------------------------------------------------ workload
 class Workload:
-    def __init__(self, s, lsp, seed_base):
+    """Seeded synthetic inputs of one shape (weights, a round's new rows, accepted
+    lengths, block tokens, prefix chunks) and, given the library binding `lsp`, the
+    round driven through it.  Without `lsp` (the oracle's arm) nothing of the
+    library is loaded; `device` is where the generators run (CUDA for both arms,
+    so that they see the same values)."""
+
+    def __init__(self, s, lsp, seed_base, device="cuda"):
         self.s, self.lsp = s, lsp
         self.seed_base = seed_base
-        self.w = synth.make_weights(s, seed=synth.WEIGHT_SEED, device="cuda")
-        self.ws = lsp.make_weights(self.w)
-        self.cfg = lsp.make_config(s)
+        self.device = device
+        self.w = synth.make_weights(s, seed=synth.WEIGHT_SEED, device=device)
         rows = s.B + 1
-        self.k, self.v, self.h = synth.make_features(s, rows, seed=seed_base + 5000, device="cuda")
-        self.acc = synth.make_accepted(s, seed=seed_base + 5001, device="cuda", hi=min(s.delta_max, s.B + 1))
-        self.bt = synth.make_block_tokens(s, seed=seed_base + 5002, device="cuda")
-        self.toks = torch.zeros(s.C, s.B, dtype=torch.int32, device="cuda")
-        self.logits = torch.empty(s.C, s.B, s.V, device="cuda")
-        self.sp = lsp.make_sample_params(s.temperature, seed=synth.RNG_SEED, rnd=0)
+        self.k, self.v, self.h = synth.make_features(s, rows, seed=seed_base + 5000, device=device)
+        self.acc = synth.make_accepted(s, seed=seed_base + 5001, device=device, hi=min(s.delta_max, s.B + 1))
+        self.bt = synth.make_block_tokens(s, seed=seed_base + 5002, device=device)
         self._hfold = None
+        if lsp is not None:
+            self.ws = lsp.make_weights(self.w)
+            self.cfg = lsp.make_config(s)
+            self.toks = torch.zeros(s.C, s.B, dtype=torch.int32, device=device)
+            self.logits = torch.empty(s.C, s.B, s.V, device=device)
+            self.sp = lsp.make_sample_params(s.temperature, seed=synth.RNG_SEED, rnd=0)
 
     def new_state(self):
         st = self.lsp.lsp_state_create(self.cfg)
         self.lsp.lsp_state_init(st, self.w["G"])
         return st
 
-    def fold(self, st, start, end, keep=None):
-        """Fold prefix rows [start, end) in FOLD_CHUNK-row chunks (GPU-generated, seeded)."""
+    def _chunks(self, start, end):
+        """Prefix rows [start, end) as seeded FOLD_CHUNK-row chunks: (k, v, h, rows used)."""
         s = self.s
         if self._hfold is None:
-            _, _, self._hfold = synth.make_features(s, FOLD_CHUNK, seed=self.seed_base + 7000, device="cuda")
+            _, _, self._hfold = synth.make_features(s, FOLD_CHUNK, seed=self.seed_base + 7000,
+                                                    device=self.device)
         for c0 in range(start, end, FOLD_CHUNK):
-            n = min(FOLD_CHUNK, end - c0)
             k, v, _ = synth.make_features(s, FOLD_CHUNK, seed=self.seed_base + c0 // FOLD_CHUNK,
-                                          device="cuda", with_h=False)
-            acc = torch.full((s.C,), n, dtype=torch.int32, device="cuda")
-            self.lsp.lsp_view_update(st, k, v, self._hfold, acc, rows=FOLD_CHUNK)
+                                          device=self.device, with_h=False)
+            yield k, v, self._hfold, min(FOLD_CHUNK, end - c0)
+
+    @staticmethod
+    def _kept(k, v, h, n):
+        """Request 0's share of a chunk, on the host (what the oracle folds)."""
+        return k[0:1, :, :n].cpu(), v[0:1, :, :n].cpu(), h[0:1, :, n - 1:n].cpu()
+
+    def fold(self, st, start, end, keep=None):
+        """Fold prefix rows [start, end) into `st` through the library, chunk by chunk."""
+        for k, v, h, n in self._chunks(start, end):
+            acc = torch.full((self.s.C,), n, dtype=torch.int32, device=self.device)
+            self.lsp.lsp_view_update(st, k, v, h, acc, rows=FOLD_CHUNK)
             if keep is not None:
-                keep.append((k[0:1, :, :n].cpu(), v[0:1, :, :n].cpu(),
-                             self._hfold[0:1, :, n - 1:n].cpu()))
+                keep.append(self._kept(k, v, h, n))
+
+    def prefix_rows(self, start, end):
+        """The rows `fold(..., keep=)` would keep, generated alone (nothing runs in the library)."""
+        return [self._kept(k, v, h, n) for k, v, h, n in self._chunks(start, end)]
 
     def round(self, st):
         self.lsp.lsp_view_update(st, self.k, self.v, self.h, self.acc)
@@ -517,20 +538,15 @@ def workload_config(s, prefix):
             "l2": "no flush: >3 GB of weights streamed per round exceed the 129 MB L2"}
 
 
-def run_reference(args, dist):
+def run_reference(args, dist, device="cuda"):
+    """The oracle's arm: the same seeded inputs, the oracle alone on the host cores
+    (the library is neither loaded nor run)."""
     if dist.rank != 0:
         return
-    from paper_2609_37029_gb300 import build as _b
-    _b.build()
-    from paper_2609_37029_gb300 import lsp
     s = synth.SHAPES[args.config]
     prefix = args.prefix or s.prefix
-    wl = Workload(s, lsp, synth.input_seed(s) * 1000)
-    st = wl.new_state()
-    kept = []
-    wl.fold(st, 0, prefix, keep=kept)
-    torch.cuda.synchronize()
-    lsp.lsp_state_destroy(st)
+    wl = Workload(s, None, synth.input_seed(s) * 1000, device=device)
+    kept = wl.prefix_rows(0, prefix)
     leg = oracle_leg(wl, kept, args.cpu_budget, max_steps=max(1, args.steps),
                      warmup=min(args.warmup, 1))
     ms = leg["_t_req"] * s.C * 1e3
