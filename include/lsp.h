@@ -29,6 +29,19 @@
  *     word (LSP_DEV_*) read by lsp_get_error; kernels never trap.
  *   - Layouts are dense and row-major; linear weights are [out][in] with `in`
  *     contiguous (y = W x).
+ *   - Environment variables, read when a plan is made (lsp_state_create,
+ *     lsp_linear, lsp_gemm_plan_info) or a kernel is launched, change how the
+ *     work is laid out and never what it computes beyond the order of fp32
+ *     summation.  Projection GEMM: LSP_GEMM_WT (weight tiles per CTA),
+ *     LSP_GEMM_PD (L2 prefetch distance), LSP_GEMM_STAGES (ring depth cap),
+ *     LSP_GEMM_TOKG / LSP_GEMM_TOKG_GU (token groups), LSP_GEMM_OCC3 (three
+ *     CTAs per SM), LSP_GEMM_LONE_COST (split model), LSP_GEMM_CLUSTER=1
+ *     (split-K reduced in a cluster), LSP_GEMM_MCAST=1 (activation multicast),
+ *     LSP_GEMM_SCALAR_EPI (per-thread stores instead of TMA stores),
+ *     LSP_GEMM_GU_SPLITS (gate/up split over K with a separate SwiGLU);
+ *     LSP_PREFILL_CHUNK (prefill K/V stage rows: 16, 32 or 64); LSP_VIEW_FMA=1
+ *     (the FMA view-update kernel instead of the tensor-core one).  Unset is
+ *     the measured default.
  */
 #ifndef LSP_H
 #define LSP_H
