@@ -29,6 +29,11 @@
  *     word (LSP_DEV_*) read by lsp_get_error; kernels never trap.
  *   - Layouts are dense and row-major; linear weights are [out][in] with `in`
  *     contiguous (y = W x).
+ *   - Concurrency: the device work of one state (its interface, workspace and
+ *     synchronisation words) must be ordered -- one stream, or streams the
+ *     caller synchronises; calls on different states, and lsp_linear calls
+ *     with different workspaces, may overlap from any threads and streams.
+ *     The one process-wide buffer is lsp_sample_noalloc's scratch (below).
  *   - Environment variables, read when a plan is made (lsp_state_create,
  *     lsp_linear, lsp_gemm_plan_info) or a kernel is launched, change how the
  *     work is laid out and never what it computes beyond the order of fp32
