@@ -52,8 +52,6 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=150.0, help="seconds for the oracle legs")
-    ap.add_argument("--linear", default=None, metavar="M,N,K[,splits]",
-                    help="profiling probe: time the projection GEMM alone (lsp_linear, bf16) and exit")
     return ap.parse_args()
 
 
@@ -705,39 +703,8 @@ def run_ours(args, dist):
     lsp.lsp_state_destroy(st)
 
 
-def linear_probe(spec, launches=4):
-    """Time `launches` lsp_linear calls of one bf16 shape, each after a 256 MB L2
-    flush (the launch to capture under ncu is the third)."""
-    from paper_2609_37029_gb300 import lsp
-    dims = [int(v) for v in spec.split(",")]
-    M, N, K = dims[:3]
-    splits = dims[3] if len(dims) > 3 else 1
-    g = torch.Generator(device="cuda").manual_seed(1)
-    X = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
-    W = (torch.randn(N, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
-    Y = torch.empty(M, N, device="cuda")
-    nb = lsp.lsp_linear_workspace_bytes(M, N, splits) if splits > 1 else 0
-    ws = torch.zeros(max(nb, 4), dtype=torch.uint8, device="cuda") if nb else None
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    us = []
-    for _ in range(launches):
-        flush.zero_()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        lsp.lsp_linear(X, W, Y, M, N, K, lsp.LSP_DTYPE_BF16, splits, ws, nb)
-        e1.record()
-        torch.cuda.synchronize()
-        us.append(e0.elapsed_time(e1) * 1e3)
-    ref = X[:64].float() @ W.float().T
-    err = float((Y[:64] - ref).abs().max() / ref.abs().max())
-    print(json.dumps({"linear": [M, N, K, splits], "us": [round(u, 1) for u in us], "relerr": err}))
-    return err < 1e-4
-
-
 def main():
     args = parse_args()
-    if args.linear:
-        sys.exit(0 if linear_probe(args.linear) else 1)
     dist = Dist()
     try:
         if args.impl == "reference":

@@ -34,19 +34,11 @@
  *     caller synchronises; calls on different states, and lsp_linear calls
  *     with different workspaces, may overlap from any threads and streams.
  *     The one process-wide buffer is lsp_sample_noalloc's scratch (below).
- *   - Environment variables, read when a plan is made (lsp_state_create,
- *     lsp_linear, lsp_gemm_plan_info) or a kernel is launched, change how the
+ *   - Environment variables, read when a kernel is launched, change how the
  *     work is laid out and never what it computes beyond the order of fp32
- *     summation.  Projection GEMM: LSP_GEMM_WT (weight tiles per CTA),
- *     LSP_GEMM_PD (L2 prefetch distance), LSP_GEMM_STAGES (ring depth cap),
- *     LSP_GEMM_TOKG / LSP_GEMM_TOKG_GU (token groups), LSP_GEMM_OCC3 (three
- *     CTAs per SM), LSP_GEMM_LONE_COST (split model), LSP_GEMM_CLUSTER=1
- *     (split-K reduced in a cluster), LSP_GEMM_MCAST=1 (activation multicast),
- *     LSP_GEMM_SCALAR_EPI (per-thread stores instead of TMA stores),
- *     LSP_GEMM_GU_SPLITS (gate/up split over K with a separate SwiGLU);
- *     LSP_PREFILL_CHUNK (prefill K/V stage rows: 16, 32 or 64); LSP_VIEW_FMA=1
- *     (the FMA view-update kernel instead of the tensor-core one).  Unset is
- *     the measured default.
+ *     summation: LSP_PREFILL_CHUNK (prefill K/V stage rows: 16, 32 or 64);
+ *     LSP_VIEW_FMA=1 (the FMA view-update kernel instead of the tensor-core
+ *     one).  Unset is the measured default.
  */
 #ifndef LSP_H
 #define LSP_H
@@ -259,13 +251,17 @@ int lsp_sample(lsp_state* st, const float* base_logits, const int32_t* prev_toke
  *   dev_error: optional device uint32 that receives LSP_DEV_* bits (OR-ed in;
  *   NULL skips error reporting).
  * Scratch: a fixed 512 KiB __device__ array inside the library, held by every
- * GPU that loads it until the process exits; a call needs 16 * (2 * SMs) * C
- * bytes of it and returns LSP_ERR_SHAPE beyond that.  The first call on a
- * device looks up the array's device address and the SM count; make that
- * first call before any stream capture on the device.  Every call shares the
- * array: calls that overlap on the GPU (other streams or threads) race, so
- * the caller must serialise them.  Allocates nothing and calls no allocating
- * CUDA or library routine. */
+ * GPU that loads it until the process exits.  A call needs
+ *   align256(16 * nblk * C) + align256(2048 * B + 4 * B) bytes of it,
+ * with nblk = min(2 * SMs, 512) and align256(x) = x rounded up to 256, and
+ * returns LSP_ERR_SHAPE beyond 512 KiB (on 152 SMs: C = 16 fits B <= 217,
+ * C = 64 fits B <= 103).  The first successful call on a device looks up the
+ * array's device address and the SM count (a failed lookup is retried by the
+ * next call); make that first call before any stream capture on the device.
+ * Every call shares the array: calls that overlap on the GPU (other streams
+ * or threads) race, so the caller must serialise them.  The step counters are
+ * cleared on the caller's stream before each launch.  Allocates nothing and
+ * calls no allocating CUDA or library routine. */
 int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_token, const void* Ec,
                        const void* Wc, int dtype, int C, int B, int V, int rc,
                        const lsp_sample_params* sp, int32_t* out_tokens, float* out_logits,
@@ -314,26 +310,16 @@ int lsp_verify(lsp_state* st, const float* target_logits, const float* draft_log
  * every projection of lsp_draft uses), for checking it on its own.
  *   X device dtype [M][K]; W device dtype [N][K]; Y device float [M][N].
  *   M <= 512; K * element size a multiple of 16 bytes.
- *   splits: split-K factor (1..16, at most the number of K blocks).  The
- *   kernel writes fp32 partial sums to `workspace` (device, at
+ *   splits: split-K factor (1..16, at most the number of K blocks).  With
+ *   splits > 1 the kernel writes fp32 partial sums to `workspace` (device, at
  *   least lsp_linear_workspace_bytes(M, N, splits) bytes) and a second kernel
- *   sums them in split order into Y.  With the environment variable
- *   LSP_GEMM_CLUSTER=1 and splits 2, 4 or 8 instead, the split CTAs of each
- *   128-row weight tile form a thread-block cluster that sums its partials in
- *   distributed shared memory, in split order, and writes Y (workspace unused;
- *   the drafter's projections then reduce the same way).
- *   Two more variables change how the work is laid out, never the result:
- *   LSP_GEMM_TOKG=G (2..4) splits the M tokens over G CTAs per weight tile
- *   (LSP_GEMM_TOKG_GU for the drafter's SwiGLU gate/up projection alone,
- *   which takes 2 by default at M >= 128 when its tiles fill less than one
- *   wave), and LSP_GEMM_MCAST=1 pairs CTAs of adjacent weight tiles in
- *   clusters that share each activation tile by TMA multicast. */
+ *   sums them in split order into Y; with splits == 1 Y is written directly
+ *   and `workspace` may be NULL. */
 size_t lsp_linear_workspace_bytes(int M, int N, int splits);
 
 /* Diagnostic, host only (needs no GPU): the launch plan the drafter's
  * projection GEMM takes for M token rows, N output features and reduction
- * length K on a device with num_sms SMs, under the current environment
- * (the LSP_GEMM_* variables above).
+ * length K on a device with num_sms SMs.
  *   swiglu = 0: a projection whose fp32 split-K partials a consumer sums
  *   (the q/k/v, o, down and boundary-fusion projections); swiglu = 1: the
  *   fused gate/up projection with N = F (gate and up each [F][K]).

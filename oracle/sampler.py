@@ -11,7 +11,9 @@ Readings where the paper is silent:
   g_v = -log(-log u_v), u_v = ((x_v >> 9) + 1/2) * 2^-23 and x_v the Philox word
   of (request b, step i, round, v).  T = 0 is greedy: y = argmax_v z_v.
 * Ties go to the lowest vocabulary index.  The argmax decision is taken on the
-  score rounded to fp32, the precision the CUDA sampler decides in.
+  score rounded to fp32: the paper fixes no precision for it, so the oracle
+  decides in the CUDA sampler's.  Positions are compared only where the fp64
+  top-1/top-2 margin exceeds 1e-2, where an fp64 argmax would agree.
 """
 from __future__ import annotations
 

@@ -6,9 +6,9 @@
 // large weight.  The kernel therefore puts 128 weight rows on the UMMA M axis
 // and the tokens on its N axis ("swap AB"): D^T[n][m] = sum_k W[n][k] X[m][k].
 //
-//   warp 0      TMA producer: `wt` 128 x BK weight tiles and the CTA's
+//   warp 0      TMA producer: the CTA's 128 x BK weight tile and its
 //               m_pad x BK activation tile per stage into an S-deep mbarrier
-//               ring, plus L2 prefetches of the weight tiles `pd` stages ahead
+//               ring, plus an L2 prefetch of the next stage's weight tile
 //   warp 1      TMEM allocation and the single-thread tcgen05.mma issue (a
 //               lean loop: this one thread's instructions set the issue rate)
 //   warps 2-5   epilogue: tcgen05.ld of the fp32 accumulators, the fused
@@ -20,9 +20,7 @@
 // Grid: x = weight-tile CTAs x token groups (a group's CTAs share the weight
 // tile, each over m_pad consecutive tokens; the SwiGLU gate/up projection
 // takes two groups when its tiles fill under one wave of two CTAs per SM),
-// y = split-K.  Kept opt-in after measuring slower: split-K reduced inside a
-// cluster (LSP_GEMM_CLUSTER=1) and activation multicast across CTA pairs
-// (LSP_GEMM_MCAST=1).
+// y = split-K.
 //
 // Launched as a programmatic dependent: before the preceding kernel finishes,
 // the producer already streams this launch's weights (L2 prefetch and the
@@ -54,6 +52,9 @@ template <> struct GemmType<float> {
 };
 
 constexpr uint32_t kTileBytes = kTileRows * 128;   // one weight tile per stage: 16 KB
+// L2 prefetch distance of the weight stream, in k-blocks (one ahead: 318 -> 281 us at the
+// LM-head shape; longer distances were slower)
+constexpr int kPrefetchDist = 1;
 
 // The epilogue's named barrier (id 1) counts exactly the four epilogue warps
 // 2-5: any other warp taking that branch would leave bar.sync waiting forever.
@@ -121,8 +122,8 @@ constexpr uint32_t kXchgBytes = 17408;                        // 128 x 33 floats
 // reaches the next token group's rows.
 template <typename T>
 __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensorMap* to, uint8_t* smem,
-                                             uint32_t lane_base, int ntl, int tile0, int tok0,
-                                             int split, int r) {
+                                             uint32_t lane_base, int tile, int tok0, int split,
+                                             int r) {
   const bool swiglu = p.mode == EPI_SWIGLU;
   const bool f32out = p.mode == EPI_F32 || p.mode == EPI_PARTIAL;
   const int es = f32out ? 4 : (int)sizeof(T);
@@ -134,10 +135,10 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
   const bool issuer = r == 0;
   const int m_end = min(p.m_pad, p.M - tok0);                 // > 0: no token group is empty
   int chunk = 0;
-  for (int w = 0; w < ntl; ++w) {
+  {
     for (int m0 = 0; m0 < m_end; m0 += TT, ++chunk) {       // no store box starts past row M
       float v[32];
-      const uint32_t col = (uint32_t)(w * p.m_pad + m0);
+      const uint32_t col = (uint32_t)m0;
       if (TT == 32) tmem_ld32(lane_base + col, v);
       else tmem_ld16(lane_base + col, v);
       uint8_t* stg = stg0 + (chunk & 1) * buf_bytes;
@@ -173,94 +174,12 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
       fence_proxy_async_smem();
       named_bar(1, kEpilogueThreads);
       if (issuer) {
-        tma_store_3d(to, smem_u32(stg), (tile0 + w) * cols, tok0 + m0, split);
+        tma_store_3d(to, smem_u32(stg), tile * cols, tok0 + m0, split);
         bulk_commit();
       }
     }
   }
   if (issuer) bulk_wait_read<0>();                            // staging smem is released at exit
-}
-
-// Split-K reduction inside the cluster (all threads of the CTA call it the
-// same number of times; one weight tile per CTA).  Pass by pass over
-// cr_tok-token chunks of the accumulator: the epilogue warps dump their TMEM
-// rows into this CTA's idle stage ring as [token][128 rows] fp32; after a
-// cluster barrier, the CTA of cluster rank k sums the k-th token slice of the
-// chunk over the split CTAs in split order (deterministic) through
-// distributed shared memory and writes the final output; a second barrier
-// frees the dumps for the next pass.
-template <typename T>
-__device__ __forceinline__ void epilogue_cluster(const GemmParams& p, uint8_t* smem, uint32_t tmem_base,
-                                                 int tile, bool have_acc) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int s = p.splits;
-  const uint32_t rank = cluster_ctarank();
-  float* dump = reinterpret_cast<float*>(smem);
-  const uint32_t dump_u32 = smem_u32(dump);
-  const bool swiglu = p.mode == EPI_SWIGLU;
-  const bool f32out = p.mode == EPI_F32 || p.mode == EPI_PARTIAL;
-  const int q = warp & 3, r = q * 32 + lane;                  // TMEM lane = weight row
-  const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
-  const int groups = swiglu ? 16 : 32;                        // float4 row groups per token
-  for (int p0 = 0; p0 < p.m_pad; p0 += p.cr_tok) {
-    const int np = min(p.cr_tok, p.m_pad - p0);
-    if (warp >= 2 && have_acc) {
-      for (int c0 = 0; c0 < np; c0 += 16) {
-        float v[16];
-        tmem_ld16(lane_base + (uint32_t)(p0 + c0), v);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) dump[(c0 + j) * kTileRows + r] = v[j];
-      }
-    }
-    cluster_sync_all();
-    const int tl = (np + s - 1) / s;
-    const int t0 = (int)rank * tl, t1 = min(t0 + tl, np);
-    for (int g = threadIdx.x; g < (t1 - t0) * groups; g += blockDim.x) {
-      const int t = t0 + g / groups, r4 = (g % groups) * 4;
-      const int m = p0 + t;
-      if (m >= p.M) continue;
-      // every peer's value in flight at once, then the sum in split order
-      float4 xa[kMaxClusterSplits], xu[kMaxClusterSplits];
-      const uint32_t off = dump_u32 + (uint32_t)((t * kTileRows + r4) * 4);
-#pragma unroll
-      for (int k = 0; k < kMaxClusterSplits; ++k)
-        if (k < s) {
-          xa[k] = ld_dsmem_f4(off, (uint32_t)k);
-          if (swiglu) xu[k] = ld_dsmem_f4(off + 64 * 4, (uint32_t)k);
-        }
-      float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
-#pragma unroll
-      for (int k = 0; k < kMaxClusterSplits; ++k)
-        if (k < s) {
-          a.x += xa[k].x; a.y += xa[k].y; a.z += xa[k].z; a.w += xa[k].w;
-          if (swiglu) { u.x += xu[k].x; u.y += xu[k].y; u.z += xu[k].z; u.w += xu[k].w; }
-        }
-      const float av[4] = {a.x, a.y, a.z, a.w}, uv[4] = {u.x, u.y, u.z, u.w};
-      if (swiglu) {
-        T* Y = static_cast<T*>(p.Y) + (size_t)m * p.ldy;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int f = tile * 64 + r4 + e;
-          if (f < p.N) Y[f] = from_f<T>(av[e] / (1.0f + expf(-av[e])) * uv[e]);
-        }
-      } else if (f32out) {
-        float* Y = static_cast<float*>(p.Y) + (size_t)m * p.ldy;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int n = tile * kTileRows + r4 + e;
-          if (n < p.N) Y[n] = av[e];
-        }
-      } else {
-        T* Y = static_cast<T*>(p.Y) + (size_t)m * p.ldy;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int n = tile * kTileRows + r4 + e;
-          if (n < p.N) Y[n] = from_f<T>(av[e]);
-        }
-      }
-    }
-    cluster_sync_all();
-  }
 }
 
 template <typename T, int kOcc>
@@ -273,7 +192,7 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int S = p.stages;
-  const uint32_t stage_a = (uint32_t)p.wt * kTileBytes;
+  const uint32_t stage_a = kTileBytes;
   const uint32_t stage_bytes = stage_a + (uint32_t)p.m_pad * 128;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 1);
@@ -281,32 +200,26 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // blockIdx.x = weight-tile CTA x token groups + group: the CTAs of one weight
+  // blockIdx.x = weight tile x token groups + group: the CTAs of one weight
   // tile are adjacent, so they run together and share the tile through L2
   const int group = (int)blockIdx.x % p.tok_groups;
-  const int tile0 = ((int)blockIdx.x / p.tok_groups) * p.wt;
+  const int tile = (int)blockIdx.x / p.tok_groups;
   const int tok0 = group * p.m_pad;                            // first token row of this CTA
-  const int ntl = min(p.wt, p.n_tiles - tile0);                // weight tiles of this CTA
   const int split = blockIdx.y;
   const int kb0 = (int)((long long)split * p.kblocks / p.splits);
   const int kb1 = (int)((long long)(split + 1) * p.kblocks / p.splits);
   const int nk = kb1 - kb0;
-  const uint32_t expect = (uint32_t)ntl * kTileBytes + (uint32_t)p.m_pad * 128;
+  const uint32_t expect = kTileBytes + (uint32_t)p.m_pad * 128;
 
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
   const uint32_t acc_bar = bar0 + 8u * (2 * S);
 
-  // Activation multicast (p.mcast): the two CTAs of a cluster hold adjacent
-  // weight tiles and the same tokens; each loads half of every activation box
-  // into both, and a stage is refilled only after both released it.
-  const bool mcast = p.mcast != 0;
-  const uint32_t crank = mcast ? cluster_ctarank() : 0u;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), mcast ? 2 : 1);
+      mbar_init(empty_bar(s), 1);
     }
     mbar_init(acc_bar, 1);
     *s_abort = 0;
@@ -318,7 +231,6 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), (uint32_t)p.tmem_cols);
   tc_fence_before();
   __syncthreads();
-  if (mcast) cluster_sync_all();          // the peer's barriers exist before anything lands in them
   tc_fence_after();
   griddep_launch();
   const uint32_t tmem_base = *tmem_slot;
@@ -329,54 +241,39 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     // a weight tile read by one CTA goes first; shared by token groups, it stays
     const uint64_t pol_w = p.tok_groups > 1 ? policy_evict_normal() : policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
-    // weight tile w of this CTA: segment (tensor map) and first row within it
-    auto a_seg = [&](int w) {
-      const int tile = tile0 + w;
-      return (p.nseg > 2 && tile >= p.seg_tile0[2]) ? 2 : (p.nseg > 1 && tile >= p.seg_tile0[1]) ? 1 : 0;
-    };
-    auto a_map = [&](int seg) { return seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2); };
+    // the tile's tensor map (segment) and first row within it
+    const int seg = (p.nseg > 2 && tile >= p.seg_tile0[2]) ? 2 : (p.nseg > 1 && tile >= p.seg_tile0[1]) ? 1 : 0;
+    const CUtensorMap* amap = seg == 0 ? &ta0 : (seg == 1 ? &ta1 : &ta2);
+    const int arow = p.mode == EPI_SWIGLU ? tile * 64 : (tile - p.seg_tile0[seg]) * kTileRows;
     auto load_a = [&](int i, uint32_t sa, uint32_t bar) {
       const int kx = (kb0 + i) * G::BK;
-      for (int w = 0; w < ntl; ++w) {
-        if (p.mode == EPI_SWIGLU) {
-          const int row = (tile0 + w) * 64;
-          tma_load_2d(sa + w * kTileBytes, &ta0, bar, kx, row, pol_w);
-          tma_load_2d(sa + w * kTileBytes + 64 * 128, &ta1, bar, kx, row, pol_w);
-        } else {
-          const int seg = a_seg(w);
-          tma_load_2d(sa + w * kTileBytes, a_map(seg), bar, kx, (tile0 + w - p.seg_tile0[seg]) * kTileRows,
-                      pol_w);
-        }
+      if (p.mode == EPI_SWIGLU) {                  // 64 gate rows, then the 64 matching up rows
+        tma_load_2d(sa, &ta0, bar, kx, arow, pol_w);
+        tma_load_2d(sa + 64 * 128, &ta1, bar, kx, arow, pol_w);
+      } else {
+        tma_load_2d(sa, amap, bar, kx, arow, pol_w);
       }
     };
     auto prefetch_a = [&](int i) {
       if (group != 0) return;                // one CTA of the tile prefetches it
       const int kx = (kb0 + i) * G::BK;
-      for (int w = 0; w < ntl; ++w) {
-        if (p.mode == EPI_SWIGLU) {
-          tma_prefetch_l2(&ta0, kx, (tile0 + w) * 64);
-          tma_prefetch_l2(&ta1, kx, (tile0 + w) * 64);
-        } else {
-          const int seg = a_seg(w);
-          tma_prefetch_l2(a_map(seg), kx, (tile0 + w - p.seg_tile0[seg]) * kTileRows);
-        }
+      if (p.mode == EPI_SWIGLU) {
+        tma_prefetch_l2(&ta0, kx, arow);
+        tma_prefetch_l2(&ta1, kx, arow);
+      } else {
+        tma_prefetch_l2(amap, kx, arow);
       }
     };
     auto load_b = [&](int i, uint32_t sb, uint32_t bar) {
       const int kx = (kb0 + i) * G::BK;
-      for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
-        if (mcast) {                          // rows [crank * bn/2, +bn/2) of the box, to both CTAs
-          const int h = p.bn / 2, r0 = tt * p.bn + (int)crank * h;
-          tma_load_2d_mc(sb + (uint32_t)(r0 * 128), &tb, bar, kx, tok0 + r0, (uint16_t)0x3, pol_x);
-        } else {
-          tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, bar, kx, tok0 + tt * p.bn, pol_x);
-        }
-      }
+      for (int tt = 0; tt < p.n_tok_tiles; ++tt)
+        tma_load_2d(sb + (uint32_t)(tt * p.bn * 128), &tb, bar, kx, tok0 + tt * p.bn, pol_x);
     };
-    // Weights do not depend on the preceding kernel: start streaming them now.
+    // Weights do not depend on the preceding kernel: start streaming them now
+    // (the first stages, and an L2 prefetch one k-block ahead of the ring).
     int next_pf = 0;
     const int pre = min(S, nk);
-    while (next_pf < min(p.pd, nk)) prefetch_a(next_pf++);
+    while (next_pf < min(kPrefetchDist, nk)) prefetch_a(next_pf++);
     for (int i = 0; i < pre; ++i) {
       mbar_expect_tx(full_bar(i), expect);
       load_a(i, smem_u32(smem + (size_t)i * stage_bytes), full_bar(i));
@@ -390,7 +287,7 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     uint32_t ph = (uint32_t)(pre / S) & 1u;
     const uint32_t ring0 = smem_u32(smem);
     for (int i = pre; i < nk; ++i) {
-      while (next_pf < nk && next_pf < i + p.pd) prefetch_a(next_pf++);
+      while (next_pf < nk && next_pf < i + kPrefetchDist) prefetch_a(next_pf++);
       if (!mbar_wait(empty_bar(s), ph ^ 1u, p.err)) { *s_abort = 1; break; }
       mbar_expect_tx(full_bar(s), expect);
       const uint32_t sa = ring0 + (uint32_t)s * stage_bytes;
@@ -408,7 +305,7 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     // field never carries), and the stage and phase advance by counters.
     const uint32_t idesc = make_idesc(p.bn, G::FMT);
     const uint32_t ring0 = smem_u32(smem);
-    const bool one_tile = ntl == 1 && p.n_tok_tiles == 1;
+    const bool one_tile = p.n_tok_tiles == 1;
     int s = 0;
     uint32_t ph = 0;
     for (int i = 0; i < nk; ++i) {
@@ -428,22 +325,18 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
       } else {
 #pragma unroll
         for (int kk = 0; kk < G::BK / G::UK; ++kk) {
-          for (int w = 0; w < ntl; ++w) {
-            const uint64_t ad = ad0 + (uint64_t)((w * kTileBytes + kk * 32) >> 4);
-            for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
-              const uint64_t bd = bd0 + (uint64_t)((tt * p.bn * 128 + kk * 32) >> 4);
-              const uint32_t col = (uint32_t)((w * p.n_tok_tiles + tt) * p.bn);
-              const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-              if constexpr (sizeof(T) == 2)
-                umma_f16(tmem_base + col, ad, bd, idesc, acc);
-              else
-                umma_tf32(tmem_base + col, ad, bd, idesc, acc);
-            }
+          const uint64_t ad = ad0 + (uint64_t)((kk * 32) >> 4);
+          for (int tt = 0; tt < p.n_tok_tiles; ++tt) {
+            const uint64_t bd = bd0 + (uint64_t)((tt * p.bn * 128 + kk * 32) >> 4);
+            const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+            if constexpr (sizeof(T) == 2)
+              umma_f16(tmem_base + (uint32_t)(tt * p.bn), ad, bd, idesc, acc);
+            else
+              umma_tf32(tmem_base + (uint32_t)(tt * p.bn), ad, bd, idesc, acc);
           }
         }
       }
-      if (mcast) umma_commit_mc(empty_bar(s), (uint16_t)0x3);
-      else umma_commit(empty_bar(s));
+      umma_commit(empty_bar(s));
       if (++s == S) { s = 0; ph ^= 1u; }
     }
     umma_commit(acc_bar);
@@ -458,18 +351,15 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     tc_fence_after();
     named_bar(1, kEpilogueThreads);
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
-    if (p.creduce) {
-      // reduced across the cluster below, by the whole CTA
-    } else if (*s_abort == 0 && p.tma_out) {
-      epilogue_tma<T>(p, &to, smem, lane_base, ntl, tile0, tok0, split, r);
+    if (*s_abort == 0 && p.tma_out) {
+      epilogue_tma<T>(p, &to, smem, lane_base, tile, tok0, split, r);
     } else if (*s_abort == 0) {
-      for (int w = 0; w < ntl; ++w)
-        for (int tt = 0; tt < p.n_tok_tiles; ++tt)
-          for (int c0 = 0; c0 < p.bn; c0 += 16) {
-            float v[16];
-            tmem_ld16(lane_base + (uint32_t)((w * p.n_tok_tiles + tt) * p.bn + c0), v);
-            emit_chunk<T>(p, tile0 + w, split, r, tok0 + tt * p.bn + c0, v, xchg);
-          }
+      for (int tt = 0; tt < p.n_tok_tiles; ++tt)
+        for (int c0 = 0; c0 < p.bn; c0 += 16) {
+          float v[16];
+          tmem_ld16(lane_base + (uint32_t)(tt * p.bn + c0), v);
+          emit_chunk<T>(p, tile, split, r, tok0 + tt * p.bn + c0, v, xchg);
+        }
     }
   }
 
@@ -479,23 +369,6 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     // A wait gave up: let every TMA copy this CTA issued land before exit.
     for (int i = (issued > S ? issued - S : 0); i < issued; ++i)
       mbar_wait(full_bar(i % S), (uint32_t)(i / S) & 1u, p.err);
-  }
-  if (mcast) {
-    // The peer's last releases arrive on this CTA's barriers: take them all
-    // before either CTA of the pair exits.
-    if (warp == 0 && lane == 0 && *s_abort == 0)
-      for (int i = (nk > S ? nk - S : 0); i < nk; ++i)
-        if (!mbar_wait(empty_bar(i % S), (uint32_t)(i / S) & 1u, p.err)) break;
-    __syncwarp();
-    cluster_sync_all();
-  }
-  if (p.creduce) {
-    // the stage ring is idle: every load landed before the last MMA was issued
-    // (or, after an abort, in the drain above); the dumps reuse it
-    __syncthreads();
-    tc_fence_after();
-    epilogue_cluster<T>(p, smem, tmem_base, tile0, *s_abort == 0);
-    tc_fence_before();
   }
   if (warp == 1) {
     tc_fence_after();
@@ -595,97 +468,70 @@ int gemm_group_rows(int M, int G) {
 
 static constexpr int kSmemBudget = 227 * 1024;
 
-// Tuning overrides for measurement sweeps: LSP_GEMM_WT (weight tiles per CTA),
-// LSP_GEMM_PD (L2 prefetch distance in k-blocks), LSP_GEMM_STAGES,
-// LSP_GEMM_TOKG (token groups; LSP_GEMM_TOKG_GU for the SwiGLU gate/up
-// projection alone).  Unset or non-positive values keep the defaults; the
-// values never change results.
-static int tuning(const char* name) {
-  const char* v = std::getenv(name);
-  return v ? std::atoi(v) : 0;
-}
-
 // Two 2-stage CTAs per SM keep the tensor pipe fed from two MMA issuers and
 // overlap one CTA's prologue/epilogue with the other's weight stream; the pair
 // must fit one SM's shared memory and TMEM.
-static bool two_per_sm_fits(int wt, int m_pad) {
-  const int stage_bytes = wt * (int)kTileBytes + m_pad * 128;
-  return 2 * stage_bytes + 2048 <= kSmemBudget / 2 && 2 * wt * m_pad <= 512;
+static bool two_per_sm_fits(int m_pad) {
+  const int stage_bytes = (int)kTileBytes + m_pad * 128;
+  return 2 * stage_bytes + 2048 <= kSmemBudget / 2 && 2 * m_pad <= 512;
 }
 
-static bool use_two_per_sm(long long ctas, int num_sms, int wt, int m_pad) {
-  return ctas * 4 >= (long long)num_sms * 5 && two_per_sm_fits(wt, m_pad);
+static bool use_two_per_sm(long long ctas, int num_sms, int m_pad) {
+  return ctas * 4 >= (long long)num_sms * 5 && two_per_sm_fits(m_pad);
 }
 
 // Three 2-stage CTAs per SM (shared memory incl. the 1 KB each CTA reserves,
 // TMEM columns, and the kernel instance bounded to 3 x 192 threads' registers)
-// when there are enough CTAs to give most SMs a third.  Used with token groups
-// (or, for sweeps, LSP_GEMM_OCC3=1).
+// when token groups give enough CTAs for most SMs to hold a third.
 constexpr int kSmemPerSm = 228 * 1024;
-static bool three_per_sm_fits(int wt, int m_pad, int groups) {
-  if (groups < 2 && tuning("LSP_GEMM_OCC3") <= 0) return false;
+static bool three_per_sm_fits(int m_pad, int groups) {
+  if (groups < 2) return false;
   int cols = 32;
-  while (cols < wt * m_pad) cols *= 2;
-  const int stage_bytes = wt * (int)kTileBytes + m_pad * 128;
+  while (cols < m_pad) cols *= 2;
+  const int stage_bytes = (int)kTileBytes + m_pad * 128;
   return 3 * (2 * stage_bytes + 1280 + 1024) <= kSmemPerSm && 3 * cols <= 512;
 }
 
-static bool use_three_per_sm(long long ctas, int num_sms, int wt, int m_pad, int groups) {
-  return ctas >= 2LL * num_sms && three_per_sm_fits(wt, m_pad, groups);
+static bool use_three_per_sm(long long ctas, int num_sms, int m_pad, int groups) {
+  return ctas >= 2LL * num_sms && three_per_sm_fits(m_pad, groups);
 }
 
 // Token groups: the CTAs of a weight tile split the M tokens G ways (each
 // streams the tile; the copies after the first come from L2).  Smaller stages
-// let three CTAs share an SM.  Default: two groups for the SwiGLU gate/up
-// projection when its tiles fill less than one wave of two CTAs per SM and two
-// groups reach three per SM (Qwen3-8B round, M = 256, 192 tiles: gate/up 368 ->
-// 359 us per round, round 1.243 -> 1.231 ms); one otherwise (the other
-// projections and the LM head measured slower with two: more CTAs re-stream
-// each weight tile for the same work).
+// let three CTAs share an SM.  Two groups for the SwiGLU gate/up projection
+// when its tiles fill at least one wave of one CTA per SM but less than one
+// of two and the token count allows it (Qwen3-8B round, M = 256, 192 tiles:
+// gate/up 368 -> 359 us per round, round 1.243 -> 1.231 ms); one otherwise
+// (every other projection and the LM head measured slower with two or three:
+// more CTAs re-stream each weight tile for the same work).
 static int token_groups(int M, int mode, int n_tiles, int num_sms) {
-  int req = mode == EPI_SWIGLU && M >= 128 && n_tiles <= 2 * num_sms && n_tiles >= num_sms ? 2 : 1;
-  if (tuning("LSP_GEMM_TOKG") > 0) req = tuning("LSP_GEMM_TOKG");
-  if (mode == EPI_SWIGLU && tuning("LSP_GEMM_TOKG_GU") > 0) req = tuning("LSP_GEMM_TOKG_GU");
-  int g = std::min(std::min(std::max(1, req), 4), std::max(1, M / 16));
-  // every group holds at least one token row
-  for (; g > 1; --g) {
-    int bn, ntt;
-    token_tiling((M + g - 1) / g, &bn, &ntt);
-    if ((g - 1) * bn * ntt < M) break;
-  }
-  return g;
+  const int g = mode == EPI_SWIGLU && M >= 128 && n_tiles <= 2 * num_sms && n_tiles >= num_sms ? 2 : 1;
+  if (g == 1) return 1;
+  int bn, ntt;
+  token_tiling((M + g - 1) / g, &bn, &ntt);
+  return (g - 1) * bn * ntt < M ? g : 1;     // every group holds at least one token row
 }
 
 // Split-K factor from a cost model in units of one k-block of one of two
-// co-resident CTAs (~1.6 us measured at M = 256): waves x (k-blocks per CTA +
-// fixed per-CTA cost) + the cost of combining the splits (fixed_cost +
-// per_split_cost per split: the consumer's re-read of fp32 partials from L2,
-// or the in-cluster reduction).  A lone CTA on an SM, with its deeper ring,
-// moves a k-block in 0.53 of that time (0.42 vs 0.80 us measured at M = 256
-// with the MMA issue loop at 0.24 us per k-block; LSP_GEMM_LONE_COST
-// overrides the factor for sweeps, and a negative value restores the fit made
-// before that loop was trimmed: 0.63 below 128 tokens, 1.0 from 128).
-static double lone_cta_cost(bool wide) {
-  const char* v = std::getenv("LSP_GEMM_LONE_COST");
-  const double f = v ? std::atof(v) : 0.53;
-  if (f < 0) return wide ? 1.0 : 0.63;
-  return f > 0 ? f : 0.53;
-}
+// co-resident CTAs (~0.8 us measured at M = 256): waves x (k-blocks per CTA +
+// fixed per-CTA cost) + the cost of combining the splits (per_split_cost per
+// split: the consumer's re-read of fp32 partials from L2).  A lone CTA on an
+// SM, with its deeper ring, moves a k-block in 0.53 of that time (0.42 vs
+// 0.80 us measured at M = 256 with the MMA issue loop at 0.24 us per k-block).
+constexpr double kLoneCtaCost = 0.53;
 
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
-                     int max_splits, int occ_max, bool wide) {
-  const double lone = lone_cta_cost(wide);
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, int max_splits,
+                     int occ_max) {
   double best = 1e30;
   int splits = 1;
   for (int s = 1; s <= std::min(max_splits, kblocks); ++s) {
-    if (max_splits == kMaxClusterSplits && s > 1 && (s & (s - 1))) continue;   // cluster sizes 2, 4, 8
     const long long ctas = (long long)n_ctas * s;
     const int occ = (occ_max >= 3 && ctas >= 2LL * num_sms) ? 3
                     : (occ_max >= 2 && ctas * 4 >= (long long)num_sms * 5) ? 2 : 1;
     const long long slots = (long long)occ * num_sms;
     const long long waves = (ctas + slots - 1) / slots;
-    const double per = (double)((kblocks + s - 1) / s) * (occ > 1 ? 1.0 : lone) + 2.0;
-    const double cost = (double)waves * per + (s > 1 ? fixed_cost + per_split_cost * s : 0.0);
+    const double per = (double)((kblocks + s - 1) / s) * (occ > 1 ? 1.0 : kLoneCtaCost) + 2.0;
+    const double cost = (double)waves * per + (s > 1 ? per_split_cost * s : 0.0);
     if (cost < best - 1e-9) { best = cost; splits = s; }
   }
   return splits;
@@ -695,59 +541,25 @@ int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost
 // model's k-block units (~1.56 us).
 double gemm_partial_cost(int M, int N) { return (double)M * N * 4.0 / 5e12 / 1.56e-6; }
 
-// Split-K reduced inside thread-block clusters, opt-in (LSP_GEMM_CLUSTER=1).
-// Measured at the Qwen3-8B drafting round it is slower than partial sums
-// through L2 (o_proj 28 vs 19.5 us per launch, round 1.41 vs 1.27 ms): the
-// distributed-shared-memory reduction runs at the tail, after the slowest
-// split, and its ~112 KB of peer reads per CTA are slow; so partials stay the
-// default and the clustered path is kept for other shapes and for testing.
-bool gemm_cluster_enabled() {
-  const char* v = std::getenv("LSP_GEMM_CLUSTER");
-  return v && v[0] == '1';
-}
-
-// Activation multicast across CTA pairs, opt-in (LSP_GEMM_MCAST=1).  Measured
-// at the Qwen3-8B drafting round it is slightly slower (LM head 267 vs 261 us,
-// round 1.269 vs 1.242 ms): halving the activation tile's L2 reads does not
-// shorten the weight stream, so each CTA loads its whole activation tile.
-bool gemm_mcast_enabled() {
-  const char* v = std::getenv("LSP_GEMM_MCAST");
-  return v && v[0] == '1';
-}
-
-// Model cost of one in-cluster reduction, k-block units: two cluster barriers
-// per pass and the distributed-shared-memory reads of the peers' dumps.
-constexpr double kClusterReduceCost = 1.5;
-
-void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt,
-                 int* groups) {
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* groups) {
   const int G = token_groups(M, mode, n_tiles, num_sms);
   if (groups) *groups = G;
   int bn, ntt;
   token_tiling((M + G - 1) / G, &bn, &ntt);
   const int m_pad = bn * ntt;
-  // one weight tile per CTA: two tiles sharing the activation tile measured slower
-  if (*wt <= 0) *wt = 1;
   const int kblocks = gemm_kblocks(K, dtype);
-  const int n_ctas = (n_tiles + *wt - 1) / *wt * G;
-  const int occ_max = three_per_sm_fits(*wt, m_pad, G) ? 3 : two_per_sm_fits(*wt, m_pad) ? 2 : 1;
-  const bool wide = m_pad >= 128;
-  if (*splits <= 0) {
-    if (gemm_cluster_enabled() && *wt == 1 && G == 1)
-      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, 0.0, kClusterReduceCost, kMaxClusterSplits,
-                                 std::min(occ_max, 2), wide);
-    else if (mode == EPI_PARTIAL)
-      *splits = gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows), 0.0, 16,
-                                 occ_max, wide);
-    else
-      *splits = 1;
-  }
+  const int n_ctas = n_tiles * G;
+  const int occ_max = three_per_sm_fits(m_pad, G) ? 3 : two_per_sm_fits(m_pad) ? 2 : 1;
+  if (*splits <= 0)
+    *splits = mode == EPI_PARTIAL
+                  ? gemm_auto_splits(n_ctas, kblocks, num_sms, gemm_partial_cost(M, n_tiles * kTileRows), 16, occ_max)
+                  : 1;
   *splits = std::max(1, std::min(*splits, kblocks));
 }
 
 int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
               const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
-              int num_sms, int splits, int wt) {
+              int num_sms, int splits) {
   if (M < 1 || M > 512 || K < 1 || nseg < 1 || nseg > 3) return LSP_ERR_SHAPE;
   if (mode == EPI_SWIGLU && nseg != 2) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;
@@ -773,45 +585,28 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     for (int i = 0; i < nseg; ++i) p.N += seg_rows[i];
   }
   p.kblocks = gemm_kblocks(K, dtype);
-  if (wt <= 0 && tuning("LSP_GEMM_WT") > 0) wt = tuning("LSP_GEMM_WT");
   int G = 1;
-  gemm_choose(dtype, M, K, p.n_tiles, mode, num_sms, &splits, &wt, &G);
+  gemm_choose(dtype, M, K, p.n_tiles, mode, num_sms, &splits, &G);
   p.tok_groups = G;
   token_tiling((M + G - 1) / G, &p.bn, &p.n_tok_tiles);      // per token group
   p.m_pad = p.bn * p.n_tok_tiles;
-  if (wt < 1 || wt > 2 || wt * p.m_pad > 512) return LSP_ERR_SHAPE;
-  p.wt = wt;
+  if (p.m_pad > 512) return LSP_ERR_SHAPE;
   int cols = 32;
-  while (cols < wt * p.m_pad) cols *= 2;
+  while (cols < p.m_pad) cols *= 2;
   p.tmem_cols = cols;
-  const int stage_bytes = wt * (int)kTileBytes + p.m_pad * 128;
+  const int stage_bytes = (int)kTileBytes + p.m_pad * 128;
   p.stages = std::min(8, (kSmemBudget - 2048) / stage_bytes);
-  const int n_ctas = (p.n_tiles + wt - 1) / wt * G;
+  const int n_ctas = p.n_tiles * G;
   op->occ = 1;
-  if (use_three_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad, G)) {
+  if (use_three_per_sm((long long)n_ctas * splits, num_sms, p.m_pad, G)) {
     p.stages = 2;
     op->occ = 3;
-  } else if (use_two_per_sm((long long)n_ctas * splits, num_sms, wt, p.m_pad)) {
+  } else if (use_two_per_sm((long long)n_ctas * splits, num_sms, p.m_pad)) {
     p.stages = 2;
   }
-  if (tuning("LSP_GEMM_STAGES") > 0) p.stages = std::min(p.stages, tuning("LSP_GEMM_STAGES"));
   if (p.stages < 2) return LSP_ERR_SHAPE;
-  // L2 prefetch of each weight tile issued before waiting for its smem slot
-  // (distance 1: 318 -> 281 us at the LM-head shape; longer distances were slower)
-  p.pd = 1;
-  if (std::getenv("LSP_GEMM_PD")) p.pd = std::max(0, tuning("LSP_GEMM_PD"));
   p.splits = splits;
-  // split-K: reduced in a cluster of the tile's split CTAs when possible
-  // (power-of-two clusters: a cluster of 6 measured 23 co-resident clusters, not 48)
-  p.creduce = (splits == 2 || splits == 4 || splits == 8) && wt == 1 && G == 1 && gemm_cluster_enabled() ? 1 : 0;
-  if (splits > 1 && mode != EPI_PARTIAL && !p.creduce) return LSP_ERR_SHAPE;
-  p.out_splits = p.creduce ? 1 : splits;
-  // each CTA of a pair loads bn/2 rows of every activation box (a whole number
-  // of 8-row swizzle atoms: bn is a multiple of 16)
-  p.mcast = wt == 1 && G == 1 && !p.creduce && p.n_tiles >= 2 && gemm_mcast_enabled() ? 1 : 0;
-  // tokens per reduction pass: the stage ring holds a [tokens][128] fp32 dump
-  p.cr_tok = std::min(p.m_pad, (int)((size_t)p.stages * stage_bytes / (kTileRows * 4) / 16 * 16));
-  if (p.creduce && p.cr_tok < 16) return LSP_ERR_SHAPE;
+  if (splits > 1 && mode != EPI_PARTIAL) return LSP_ERR_SHAPE;
   p.Y = Y;
   p.ldy = ldy;
   p.err = err;
@@ -822,18 +617,16 @@ int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* co
     const int si = i < nseg ? i : 0;
     if ((rc = make_map(&op->a[i], dtype, W[si], K, seg_rows[si], box_rows)) != LSP_OK) return rc;
   }
-  if ((rc = make_map(&op->b, dtype, X, K, M, p.mcast ? p.bn / 2 : p.bn)) != LSP_OK) return rc;
+  if ((rc = make_map(&op->b, dtype, X, K, M, p.bn)) != LSP_OK) return rc;
   // TMA-store epilogue when the output view can be described (else per-thread stores)
   p.out_tok = (p.m_pad % 32) ? 16 : 32;
   {
     const bool f32 = mode == EPI_F32 || mode == EPI_PARTIAL || dtype == LSP_DTYPE_F32;
     const int cols = mode == EPI_SWIGLU ? 64 : kTileRows;
-    p.tma_out = make_out_map(&op->out, f32, Y, p.N, M, p.out_splits, ldy, cols, p.out_tok) == LSP_OK &&
-                std::getenv("LSP_GEMM_SCALAR_EPI") == nullptr;
+    p.tma_out = make_out_map(&op->out, f32, Y, p.N, M, splits, ldy, cols, p.out_tok) == LSP_OK;
     if (!p.tma_out) op->out = op->b;       // unused placeholder
   }
-  op->grid = dim3((unsigned)(p.mcast ? (n_ctas + 1) / 2 * 2 : n_ctas), (unsigned)splits, 1);
-  op->cluster = p.creduce ? splits : 1;
+  op->grid = dim3((unsigned)n_ctas, (unsigned)splits, 1);
   op->smem = (size_t)p.stages * stage_bytes + 1024 + 256;
   return LSP_OK;
 }
@@ -846,29 +639,8 @@ static int launch_t(const GemmOp* op, cudaStream_t s) {
     if (kOcc > 1)   // room for kOcc CTAs' shared memory on one SM
       cudaFuncSetAttribute(gemm_kernel<T, kOcc>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   });
-  if (op->cluster <= 1 && !op->p.mcast) {
-    const cudaError_t e = launch_pdl(gemm_kernel<T, kOcc>, op->grid, dim3(kGemmThreads), op->smem, s,
-                                     op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
-    return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
-  }
-  // the split CTAs of a weight tile form one cluster (grid.y == cluster size),
-  // or two adjacent weight tiles do (activation multicast)
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = op->grid;
-  cfg.blockDim = dim3(kGemmThreads);
-  cfg.dynamicSmemBytes = op->smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = op->p.mcast ? 2u : 1u;
-  attr[1].val.clusterDim.y = op->p.mcast ? 1u : (unsigned)op->cluster;
-  attr[1].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_kernel<T, kOcc>, op->a[0], op->a[1], op->a[2], op->b,
-                                           op->out, op->p);
+  const cudaError_t e = launch_pdl(gemm_kernel<T, kOcc>, op->grid, dim3(kGemmThreads), op->smem, s,
+                                   op->a[0], op->a[1], op->a[2], op->b, op->out, op->p);
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 

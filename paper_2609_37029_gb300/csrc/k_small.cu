@@ -12,10 +12,7 @@
 // residual add of the o and down projections, in split order), then
 // x / sqrt(mean(x^2) + eps) * w (Qwen3 RMSNorm) into the storage dtype that
 // the next projection's TMA reads; one CTA of up to 1024 threads per row.
-//
-// swiglu_sum_kernel: the gate/up projection split over K writes fp32 partials
-// [splits][M][2F] (gate features then up features); this sums them in split
-// order and forms silu(g) * u in the storage dtype the down projection reads.
+
 #include <algorithm>
 
 #include "common.cuh"
@@ -231,38 +228,6 @@ static cudaError_t launch_norm_t(float* x, const float* part, int splits, const 
     case 2: return launch_pdl(resid_norm_kernel<T, 2>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
     default: return cudaErrorInvalidValue;
   }
-}
-
-template <typename T>
-__global__ void __launch_bounds__(256) swiglu_sum_kernel(const float* __restrict__ part, int splits, int M,
-                                                         int F, T* __restrict__ out) {
-  griddep_launch();
-  griddep_wait();
-  const int f4 = F / 4;
-  const size_t slice = (size_t)M * 2 * F;
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * f4; i += gridDim.x * blockDim.x) {
-    const int m = i / f4, j = i - m * f4;
-    const float* g0 = part + (size_t)m * 2 * F;
-    float4 g = ld4(g0, j), u = ld4(g0 + F, j);
-    for (int s = 1; s < splits; ++s) {
-      g = add4(g, ld4(g0 + s * slice, j));
-      u = add4(u, ld4(g0 + s * slice + F, j));
-    }
-    const float4 y = make_float4(g.x / (1.0f + expf(-g.x)) * u.x, g.y / (1.0f + expf(-g.y)) * u.y,
-                                 g.z / (1.0f + expf(-g.z)) * u.z, g.w / (1.0f + expf(-g.w)) * u.w);
-    st4(out + (size_t)m * F, j, y);
-  }
-}
-
-int launch_swiglu_sum(const float* part, int splits, int M, int F, void* out, int dtype, cudaStream_t s) {
-  if (F % 4) return LSP_ERR_SHAPE;
-  const int n = M * (F / 4);
-  const dim3 grid((unsigned)std::min((n + 255) / 256, 4096));
-  const cudaError_t e =
-      dtype == LSP_DTYPE_BF16
-          ? launch_pdl(swiglu_sum_kernel<bf16>, grid, dim3(256), 0, s, part, splits, M, F, static_cast<bf16*>(out))
-          : launch_pdl(swiglu_sum_kernel<float>, grid, dim3(256), 0, s, part, splits, M, F, static_cast<float*>(out));
-  return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
 int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,

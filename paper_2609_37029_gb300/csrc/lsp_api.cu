@@ -169,22 +169,6 @@ static void partial_shapes(const lsp_config& c, int* M, int* K, int* N, int* n) 
   *n = i;
 }
 
-// Split-K factor of the gate/up projection.  1 (default): one pass with the
-// SwiGLU fused into the GEMM epilogue; > 1 (LSP_GEMM_GU_SPLITS=n): fp32
-// partials [n][M][2F] and a swiglu_sum kernel, which lets the 2F/128 weight
-// tiles fill every SM (the fused form cannot split K: the nonlinearity needs
-// the full sums).  At the Qwen3-8B round the split measured no faster (gate/up
-// 361 us per round with 3 splits, 364 fused; 2 and 4 splits slower) -- each
-// CTA's stream rate, not SM coverage, bounds it -- so fused is the default.
-static int gate_up_splits(const lsp_config& c, int num_sms) {
-  const char* v = std::getenv("LSP_GEMM_GU_SPLITS");
-  if (!v || c.F % kTileRows) return 1;               // the gate and up segments tile separately
-  int splits = std::max(1, std::atoi(v)), wt = 0;
-  const int rows[1] = {2 * c.F};
-  gemm_choose(c.dtype, c.C * c.B, c.H, gemm_tiles(EPI_PARTIAL, rows, 1), EPI_PARTIAL, num_sms, &splits, &wt);
-  return splits;
-}
-
 int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   if (!cfg || !out) return LSP_ERR_ARG;
   *out = nullptr;
@@ -231,14 +215,11 @@ int lsp_state_create(const lsp_config* cfg, lsp_state** out) {
   partial_shapes(c, pm, pk, pn, &np);
   size_t pbytes = 0;
   for (int i = 0; i < np; ++i) {
-    int splits = 0, wt = 0;
+    int splits = 0;
     const int rows[1] = {pn[i]};
-    gemm_choose(c.dtype, pm[i], pk[i], gemm_tiles(EPI_PARTIAL, rows, 1), EPI_PARTIAL, st->num_sms,
-                &splits, &wt);
+    gemm_choose(c.dtype, pm[i], pk[i], gemm_tiles(EPI_PARTIAL, rows, 1), EPI_PARTIAL, st->num_sms, &splits);
     pbytes = std::max(pbytes, (size_t)splits * pm[i] * pn[i] * sizeof(float));
   }
-  const int gus = gate_up_splits(c, st->num_sms);                   // gate | up, when split
-  if (gus > 1) pbytes = std::max(pbytes, (size_t)gus * M * 2 * c.F * sizeof(float));
   st->nblk = sample_blocks(st->num_sms);
   off = 0;
   const size_t w_x = off; off = align256(off + (size_t)M * c.H * 4);
@@ -383,9 +364,9 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
   int rc;
   auto plan = [&](GemmOp* op, const void* X, int Mx, int K, const void* const* W, const int* rows,
                   int nseg, int mode, void* Y, int ldy) {
-    const int r = gemm_plan(op, dt, X, Mx, K, W, rows, nseg, mode, Y, ldy, st->err, st->num_sms, 0, 0);
+    const int r = gemm_plan(op, dt, X, Mx, K, W, rows, nseg, mode, Y, ldy, st->err, st->num_sms, 0);
     if (r == LSP_OK && mode == EPI_PARTIAL &&
-        (size_t)op->p.out_splits * Mx * op->p.N * sizeof(float) > st->part_bytes)
+        (size_t)op->p.splits * Mx * op->p.N * sizeof(float) > st->part_bytes)
       return LSP_ERR_SHAPE;
     return r;
   };
@@ -412,15 +393,8 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
       return rc;
     const void* Wgu[2] = {lw.w_gate, lw.w_up};
     const int rgu[2] = {c.F, c.F};
-    const int gus = gate_up_splits(c, st->num_sms);
-    if (gus > 1) {
-      const int r = gemm_plan(&st->gu_op[j], c.dtype, st->xn, M, c.H, Wgu, rgu, 2, EPI_PARTIAL, st->part,
-                              2 * c.F, st->err, st->num_sms, gus, 0);
-      if (r != LSP_OK) return r;
-      if ((size_t)st->gu_op[j].p.out_splits * M * 2 * c.F * sizeof(float) > st->part_bytes) return LSP_ERR_SHAPE;
-    } else if ((rc = plan(&st->gu_op[j], st->xn, M, c.H, Wgu, rgu, 2, EPI_SWIGLU, st->act, c.F)) != LSP_OK) {
+    if ((rc = plan(&st->gu_op[j], st->xn, M, c.H, Wgu, rgu, 2, EPI_SWIGLU, st->act, c.F)) != LSP_OK)
       return rc;
-    }
     const void* Wd[1] = {lw.w_down};
     const int rd[1] = {c.H};
     if ((rc = plan(&st->down_op[j], st->act, M, c.F, Wd, rd, 1, EPI_PARTIAL, st->part, c.H)) != LSP_OK)
@@ -476,7 +450,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   // input slots + first input norm + rotary table
   CombineParams cp;
   cp.tokens = block_tokens; cp.embed = w->embed; cp.pos = w->pos; cp.mask_emb = w->mask_emb;
-  cp.c = st->h ? st->part : nullptr; cp.c_splits = st->h ? st->fuse.p.out_splits : 0; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
+  cp.c = st->h ? st->part : nullptr; cp.c_splits = st->h ? st->fuse.p.splits : 0; cp.norm_w = w->layer[0].in_norm; cp.x = st->x; cp.xn = st->xn; cp.rope = st->rope;
   cp.t = st->t; cp.err = st->err; cp.C = c.C; cp.B = c.B; cp.H = c.H; cp.V = c.V; cp.d = c.d;
   cp.eps = c.rms_eps; cp.theta = (double)c.rope_theta;
   if ((rc = launch_combine(cp, c.dtype, s)) != LSP_OK) return rc;
@@ -485,7 +459,7 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     const lsp_layer_weights& lw = w->layer[j];
     if ((rc = gemm_launch(&st->qkv_op[j], s)) != LSP_OK) return rc;
     QkvParams qp;
-    qp.part = st->part; qp.splits = st->qkv_op[j].p.out_splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
+    qp.part = st->part; qp.splits = st->qkv_op[j].p.splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
     qp.rope = st->rope; qp.out = st->qkv; qp.M = M; qp.B = c.B; qp.nq = c.nq; qp.nkv = c.nkv; qp.d = c.d;
     qp.eps = c.rms_eps;
     if ((rc = launch_qkv_finalize(qp, c.dtype, s)) != LSP_OK) return rc;
@@ -499,19 +473,16 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->o_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
-    if ((rc = launch_resid_norm(st->x, st->part, st->o_op[j].p.out_splits, lw.post_norm, st->xn, M, c.H,
+    if ((rc = launch_resid_norm(st->x, st->part, st->o_op[j].p.splits, lw.post_norm, st->xn, M, c.H,
                                 c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->gu_op[j], s)) != LSP_OK) return rc;
-    if (st->gu_op[j].p.mode == EPI_PARTIAL &&
-        (rc = launch_swiglu_sum(st->part, st->gu_op[j].p.out_splits, M, c.F, st->act, c.dtype, s)) != LSP_OK)
-      return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->down_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
     const void* next_norm = j + 1 < c.D ? w->layer[j + 1].in_norm : w->final_norm;
-    if ((rc = launch_resid_norm(st->x, st->part, st->down_op[j].p.out_splits, next_norm, st->xn, M, c.H,
+    if ((rc = launch_resid_norm(st->x, st->part, st->down_op[j].p.splits, next_norm, st->xn, M, c.H,
                                 c.rms_eps, c.dtype, s)) != LSP_OK)
       return rc;
     mark(st, ev++, s);
@@ -540,8 +511,8 @@ int lsp_gemm_plan_info(int dtype, int M, int N, int K, int swiglu, int num_sms, 
   if (dtype != LSP_DTYPE_BF16 && dtype != LSP_DTYPE_F32) return LSP_ERR_ARG;
   const int mode = swiglu ? EPI_SWIGLU : EPI_PARTIAL;
   const int rows[1] = {N};
-  int s = 0, wt = 0, g = 1;
-  gemm_choose(dtype, M, K, gemm_tiles(mode, rows, 1), mode, num_sms, &s, &wt, &g);
+  int s = 0, g = 1;
+  gemm_choose(dtype, M, K, gemm_tiles(mode, rows, 1), mode, num_sms, &s, &g);
   *splits = s;
   *tok_groups = g;
   *tokens_per_group = gemm_group_rows(M, g);
@@ -567,13 +538,13 @@ int lsp_linear(const void* X, const void* W, float* Y, int M, int N, int K, int 
   GemmOp op;
   const void* Ws[1] = {W};
   float* part = static_cast<float*>(workspace);
-  // splits <= 8: reduced inside a cluster straight into Y; else partials + a sum kernel
-  const bool in_cluster = splits == 1 || ((splits == 2 || splits == 4 || splits == 8) && gemm_cluster_enabled());
-  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, in_cluster ? EPI_F32 : EPI_PARTIAL,
-                     in_cluster ? Y : part, N, nullptr, sms, splits, 0);
+  // one split writes Y directly; more write fp32 partials that a second kernel sums
+  const bool direct = splits == 1;
+  int rc = gemm_plan(&op, dtype, X, M, K, Ws, rows, 1, direct ? EPI_F32 : EPI_PARTIAL, direct ? Y : part, N,
+                     nullptr, sms, splits);
   if (rc != LSP_OK) return rc;
   if (op.p.splits != splits) return LSP_ERR_SHAPE;
-  if ((rc = gemm_launch(&op, S(stream))) != LSP_OK || in_cluster) return rc;
+  if ((rc = gemm_launch(&op, S(stream))) != LSP_OK || direct) return rc;
   return launch_sum_partials(part, splits, (size_t)M * N, Y, S(stream));
 }
 
@@ -593,8 +564,7 @@ int lsp_round_launches(lsp_state* st) {
   // view update, fuse, combine; per layer q/k/v GEMM + finalize, attention, o, norm, gate/up, down,
   // norm; LM head; the sampler
   const int fuse = (c.flags & LSP_NO_BOUNDARY) ? 0 : 1;
-  const int gu_sum = gate_up_splits(c, st->num_sms) > 1 ? c.D : 0;   // the swiglu_sum kernels
-  return 2 + fuse + 8 * c.D + gu_sum + 1 + sample_launches(p, c.dtype);
+  return 2 + fuse + 8 * c.D + 1 + sample_launches(p, c.dtype);
 }
 
 const char* lsp_stage_name(lsp_state* st, int k) {

@@ -44,20 +44,13 @@ constexpr int kTileRows = 128;      // weight rows per tile (UMMA M)
 struct GemmParams {
   int M, N, K;          // token rows, output features, reduction length
   int kblocks, splits, n_tiles;
-  int wt;               // weight tiles per CTA (they share the activation tile)
   int mode;
   int seg_tile0[3];     // first tile index of each A segment
   int nseg;
-  int bn, n_tok_tiles, m_pad, stages, tmem_cols, pd;
+  int bn, n_tok_tiles, m_pad, stages, tmem_cols;
   int tma_out;          // 1: the epilogue stages tiles in shared memory and TMA-stores them
   int out_tok;          // tokens per staged output chunk (16 or 32)
-  int creduce;          // 1: the `splits` CTAs of a tile form a cluster and reduce split-K in
-                        //    distributed shared memory; the output is final (one slice)
-  int cr_tok;           // tokens per cluster-reduction pass (the idle stage ring holds them)
-  int out_splits;       // slices of the output the consumer sums (splits, or 1 when reduced)
   int tok_groups;       // CTAs per weight tile, each over m_pad consecutive tokens
-  int mcast;            // 1: CTA pairs (clusters of 2 along x) share each activation box by TMA
-                        //    multicast; grid.x is even (a CTA past the last tile only loads)
   void* Y;
   int ldy;
   unsigned* err;
@@ -70,36 +63,29 @@ struct GemmOp {
   GemmParams p;
   int dtype;
   dim3 grid;
-  int cluster;          // CTAs per cluster along the split axis (1: no cluster)
   int occ;              // CTAs per SM the plan sizes for: 3 picks the register-bounded instance
   size_t smem;
 };
 
 // Plan Y = X W^T where W is the row-concatenation of `nseg` weight segments
 // (each [seg_rows[i]][K]); for EPI_SWIGLU, segment 0 = gate and 1 = up, both
-// [N][K].  With splits > 1 the split-K partial sums are reduced inside a
-// thread-block cluster (splits <= kMaxClusterSplits) and every mode writes its
-// final output (EPI_PARTIAL then writes one fp32 slice: p.out_splits == 1);
-// otherwise EPI_PARTIAL writes `splits` partial sums [splits][M][ldy] for the
-// consumer to add and other modes need splits == 1.  splits <= 0 / wt <= 0
-// choose for `num_sms`.
+// [N][K].  EPI_PARTIAL writes `splits` fp32 partial sums [splits][M][ldy] for
+// the consumer to add; other modes need splits == 1.  splits <= 0 chooses
+// for `num_sms`.
 int gemm_plan(GemmOp* op, int dtype, const void* X, int M, int K, const void* const* W,
               const int* seg_rows, int nseg, int mode, void* Y, int ldy, unsigned* err,
-              int num_sms, int splits, int wt);
+              int num_sms, int splits);
 int gemm_launch(const GemmOp* op, cudaStream_t s);
-// The split-K factor and weight tiles per CTA gemm_plan uses (inputs <= 0 =
-// choose), and the token groups it splits M into (groups may be null).
-void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits, int* wt,
+// The split-K factor gemm_plan uses (input <= 0 = choose), and the token
+// groups it splits M into (groups may be null).
+void gemm_choose(int dtype, int M, int K, int n_tiles, int mode, int num_sms, int* splits,
                  int* groups = nullptr);
 int gemm_tiles(int mode, const int* seg_rows, int nseg);
 // Token rows one token group of M rows split G ways covers (a multiple of 16).
 int gemm_group_rows(int M, int G);
 // occ_max: CTAs one SM can hold (1-3) for this tile shape.
-int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, double fixed_cost,
-                     int max_splits, int occ_max, bool wide);
-constexpr int kMaxClusterSplits = 8;    // portable cluster size
-bool gemm_cluster_enabled();
-bool gemm_mcast_enabled();
+int gemm_auto_splits(int n_ctas, int kblocks, int num_sms, double per_split_cost, int max_splits,
+                     int occ_max);
 double gemm_partial_cost(int M, int N);
 int gemm_kblocks(int K, int dtype);
 // Deterministic sum of `splits` fp32 partials [splits][n] into y[n].
@@ -147,9 +133,6 @@ int launch_combine(const CombineParams& p, int dtype, cudaStream_t s);
 // x += sum_s part[s] (s < splits, fp32 [splits][M][H]); out = RMSNorm(x) * w.
 int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
                       int H, float eps, int dtype, cudaStream_t s);
-// out[m][f] = silu(g) * u with g = sum_s part[s][m][f], u = sum_s part[s][m][F + f]
-// (part fp32 [splits][M][2F]; out dtype [M][F]).
-int launch_swiglu_sum(const float* part, int splits, int M, int F, void* out, int dtype, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention
 // q | k | v of the block rows: sum of the projection's split-K partials, then

@@ -1,12 +1,10 @@
 """The projection GEMM's launch plan, host logic only (no GPU): the split-K
 factor and token groups the drafter takes at the Qwen3-8B round on a 152-SM
-GB300, what each tuning variable changes, and the token-group invariants the
-kernel relies on (every token row in exactly one group, no empty group)."""
+GB300, and the token-group invariants the kernel relies on (every token row
+in exactly one group, no empty group)."""
 import pytest
 
 GU = dict(N=12288, K=4096, swiglu=1)
-PLAN_VARS = ("LSP_GEMM_TOKG", "LSP_GEMM_TOKG_GU", "LSP_GEMM_LONE_COST", "LSP_GEMM_CLUSTER", "LSP_GEMM_WT",
-             "LSP_GEMM_MCAST")
 
 
 @pytest.fixture(scope="module")
@@ -15,12 +13,6 @@ def lsp():
     build.build()
     from paper_2609_37029_gb300 import lsp as mod
     return mod
-
-
-@pytest.fixture(autouse=True)
-def clean_env(monkeypatch):
-    for v in PLAN_VARS:
-        monkeypatch.delenv(v, raising=False)
 
 
 def plan(lsp, M, N, K, swiglu=0, sms=152, dtype=None):
@@ -36,23 +28,6 @@ def test_qwen3_8b_round_plan(lsp):
     assert plan(lsp, 256, **GU) == (1, 2, 128)              # gate/up: two token groups
 
 
-def test_lone_cta_cost_override_restores_the_earlier_fit(lsp, monkeypatch):
-    monkeypatch.setenv("LSP_GEMM_LONE_COST", "-1")
-    assert plan(lsp, 256, 6144, 4096)[0] == 6
-    assert plan(lsp, 256, 4096, 4096)[0] == 8
-
-
-def test_token_group_overrides(lsp, monkeypatch):
-    monkeypatch.setenv("LSP_GEMM_TOKG_GU", "1")
-    assert plan(lsp, 256, **GU) == (1, 1, 256)
-    monkeypatch.setenv("LSP_GEMM_TOKG", "3")                 # every projection; gate/up keeps its own
-    assert plan(lsp, 256, 6144, 4096)[1:] == (3, 96)
-    assert plan(lsp, 256, **GU)[1] == 1
-    monkeypatch.delenv("LSP_GEMM_TOKG_GU")
-    assert plan(lsp, 256, **GU)[1:] == (3, 96)
-    assert plan(lsp, 20, 6144, 4096)[1] == 1                 # fewer than 32 rows: one group
-
-
 @pytest.mark.parametrize("sms,groups", [(152, 2), (96, 2), (95, 1), (192, 2), (193, 1)])
 def test_gate_up_groups_only_for_an_underfilled_single_wave(lsp, sms, groups):
     """192 gate/up tiles: two groups when num_sms <= 192 <= 2 num_sms (at least a wave of one
@@ -61,14 +36,16 @@ def test_gate_up_groups_only_for_an_underfilled_single_wave(lsp, sms, groups):
     assert plan(lsp, 112, sms=sms, **GU)[1] == 1             # B = 7 (M = 112): one group
 
 
-@pytest.mark.parametrize("req", ["1", "2", "3", "4"])
-def test_token_groups_cover_every_row_once(lsp, monkeypatch, req):
-    monkeypatch.setenv("LSP_GEMM_TOKG", req)
+@pytest.mark.parametrize("N", [12288, 9728, 19456])
+def test_token_groups_cover_every_row_once(lsp, N):
+    """Over every token count, the gate/up plan's groups cover each row once with no
+    empty group; the other projections always take one group."""
     for M in range(1, 513):
-        _, g, rows = plan(lsp, M, 1024, 1024)
-        assert 1 <= g <= int(req) and rows % 16 == 0 and rows <= 512
+        _, g, rows = plan(lsp, M, N, 1024, swiglu=1)
+        assert 1 <= g <= 2 and rows % 16 == 0 and rows <= 512
         assert g * rows >= M > (g - 1) * rows, (M, g, rows)   # covered, last group not empty
         assert g == 1 or M >= 16 * g
+        assert plan(lsp, M, N, 1024)[1] == 1
 
 
 def test_bad_arguments(lsp):

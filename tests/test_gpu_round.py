@@ -104,41 +104,6 @@ def test_round_variants_match_oracle(lsp, variant):
     _run_round(lsp, s, 3000)
 
 
-def test_round_with_cluster_split_k(lsp, monkeypatch):
-    """The projections' split-K reduced inside thread-block clusters (opt-in) gives the
-    same round within the same tolerance."""
-    monkeypatch.setenv("LSP_GEMM_CLUSTER", "1")
-    s = synth.SMALL.with_(temperature=1.0)
-    _run_round(lsp, s, 2500)
-
-
-def test_round_with_activation_multicast(lsp, monkeypatch):
-    """The projections with each activation tile loaded once per CTA pair and multicast
-    to both (opt-in) give the same round within the same tolerance."""
-    monkeypatch.setenv("LSP_GEMM_MCAST", "1")
-    s = synth.SMALL.with_(temperature=1.0)
-    _run_round(lsp, s, 2200)
-
-
-@pytest.mark.parametrize("tokg", ["2", "4"])
-def test_round_with_token_groups(lsp, monkeypatch, tokg):
-    """Every projection with its token rows split over 2 or 4 CTAs per weight tile gives
-    the same round within the same tolerance."""
-    monkeypatch.setenv("LSP_GEMM_TOKG", tokg)
-    monkeypatch.setenv("LSP_GEMM_TOKG_GU", "2")       # gate/up with its own count
-    s = synth.SMALL.with_(temperature=1.0)
-    _run_round(lsp, s, 2000)
-
-
-@pytest.mark.parametrize("gu_splits", ["1", "3"])
-def test_round_gate_up_fused_or_split(lsp, monkeypatch, gu_splits):
-    """The gate/up projection with its SwiGLU fused into the GEMM epilogue (one pass), or
-    split over K with fp32 partials and a separate sum + SwiGLU kernel."""
-    monkeypatch.setenv("LSP_GEMM_GU_SPLITS", gu_splits)
-    s = synth.SMALL
-    _run_round(lsp, s, 1500)
-
-
 def test_round_sampled_and_short_prefix(lsp):
     """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
     s = synth.SMALL.with_(temperature=1.0)
