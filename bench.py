@@ -368,22 +368,24 @@ class Workload:
                                           device=self.device, with_h=False)
             yield k, v, self._hfold, min(FOLD_CHUNK, end - c0)
 
-    @staticmethod
-    def _kept(k, v, h, n):
-        """Request 0's share of a chunk, on the host (what the oracle folds)."""
-        return k[0:1, :, :n].cpu(), v[0:1, :, :n].cpu(), h[0:1, :, n - 1:n].cpu()
-
-    def fold(self, st, start, end, keep=None):
+    def fold(self, st, start, end):
         """Fold prefix rows [start, end) into `st` through the library, chunk by chunk."""
         for k, v, h, n in self._chunks(start, end):
             acc = torch.full((self.s.C,), n, dtype=torch.int32, device=self.device)
             self.lsp.lsp_view_update(st, k, v, h, acc, rows=FOLD_CHUNK)
-            if keep is not None:
-                keep.append(self._kept(k, v, h, n))
 
-    def prefix_rows(self, start, end):
-        """The rows `fold(..., keep=)` would keep, generated alone (nothing runs in the library)."""
-        return [self._kept(k, v, h, n) for k, v, h, n in self._chunks(start, end)]
+    def oracle_fold(self, so, ost, G, start, end, reqs):
+        """Fold the same prefix rows [start, end) of requests `reqs` into the oracle state
+        `ost` (oracle shape `so`, C = len(reqs)); nothing runs in the library.  Only each
+        chunk's last hidden row enters the boundary, so only that row is converted."""
+        import oracle
+        s = self.s
+        for k, v, h, n in self._chunks(start, end):
+            kk = k[reqs][:, :, :n].to(torch.float64).cpu().numpy()
+            vv = v[reqs][:, :, :n].to(torch.float64).cpu().numpy()
+            hl = np.broadcast_to(h[reqs][:, :, n - 1:n].to(torch.float64).cpu().numpy(),
+                                 (len(reqs), s.L, n, s.H))
+            oracle.view_update(so, ost, G, kk, vv, hl, np.full(len(reqs), n))
 
     def round(self, st):
         self.lsp.lsp_view_update(st, self.k, self.v, self.h, self.acc)
@@ -471,28 +473,35 @@ def oracle_weights(w):
     return oracle.OracleWeights(wn)
 
 
-def oracle_prefix_state(s1, ow, kept):
-    """Oracle interface of request 0 after the same prefix the GPU folded."""
-    import oracle
-    ost = oracle.state_init(s1)
-    for k, v, hlast in kept:
-        n = k.shape[2]
-        h = np.zeros((1, s1.L, n, s1.H))
-        h[:, :, n - 1] = hlast[:, :, 0].double().numpy()
-        oracle.view_update(s1, ost, ow.G, k.double().numpy(), v.double().numpy(), h, np.array([n]))
-    return ost
+class OracleRound:
+    """One whole drafting round of all C requests as the oracle computes it (view update of
+    the round's new rows, drafter forward, B-step correction + sampling per request), on
+    the state the same seeded prefix gives.  The round's inputs are converted to fp64 on
+    the host once, outside the timed calls."""
 
+    def __init__(self, wl, prefix):
+        import oracle
+        s = wl.s
+        self.s, self.wl = s, wl
+        self.reqs = list(range(s.C))
+        self.ow = oracle_weights(wl.w)
+        self.ost = oracle.state_init(s)
+        wl.oracle_fold(s, self.ost, self.ow.G, 0, prefix, self.reqs)
+        f64 = lambda t: t.detach().to(torch.float64).cpu().numpy()
+        self.k, self.v, self.h = f64(wl.k), f64(wl.v), f64(wl.h)
+        self.acc = wl.acc.cpu().numpy()
+        self.bt = wl.bt.cpu().numpy()
 
-def oracle_round(s1, ow, ost, wl):
-    """Request 0's share of one round, as the oracle computes it; returns seconds."""
-    import oracle
-    t0 = time.perf_counter()
-    oracle.view_update(s1, ost, ow.G, wl.k[0:1].double().cpu().numpy(), wl.v[0:1].double().cpu().numpy(),
-                       wl.h[0:1].double().cpu().numpy(), wl.acc[0:1].cpu().numpy())
-    bt = wl.bt[0:1].cpu().numpy()
-    z0 = oracle.draft_base_logits(s1, ost, ow, bt)
-    oracle.sample_block(z0[0], int(bt[0, 0]), ow.Ec, ow.Wc, s1.temperature, synth.RNG_SEED, 0, 0)
-    return time.perf_counter() - t0
+    def step(self):
+        """One round; returns its wall-clock seconds."""
+        import oracle
+        s, ow, ost = self.s, self.ow, self.ost
+        t0 = time.perf_counter()
+        oracle.view_update(s, ost, ow.G, self.k, self.v, self.h, self.acc)
+        z0 = oracle.draft_base_logits(s, ost, ow, self.bt)
+        for b in self.reqs:
+            oracle.sample_block(z0[b], int(self.bt[b, 0]), ow.Ec, ow.Wc, s.temperature, synth.RNG_SEED, 0, b)
+        return time.perf_counter() - t0
 
 
 def host_cores():
@@ -502,27 +511,34 @@ def host_cores():
         return os.cpu_count() or 1
 
 
-def oracle_leg(wl, kept, budget, max_steps=None, warmup=1):
+def blas_threads():
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(var):
+            return int(os.environ[var])
+    return host_cores()
+
+
+CPU_PREFIX = 4096          # prefix rows the in-run CPU baseline folds (the round's cost is prefix-free)
+
+
+def oracle_leg(wl, budget, prefix=CPU_PREFIX, warmup=1, min_s=10.0):
+    """The in-run CPU baseline: whole rounds of all C requests on the host cores after a
+    `prefix`-row prefix (the state is fixed-size, so a round costs the same at any prefix),
+    one warm-up round, then rounds until `min_s` seconds of them (or `budget`) are timed."""
     s = wl.s
-    s1 = s.with_(C=1)
-    ow = oracle_weights(wl.w)
-    ost = oracle_prefix_state(s1, ow, kept)
+    orr = OracleRound(wl, prefix)
     for _ in range(warmup):
-        oracle_round(s1, ow, ost, wl)
+        orr.step()
     times = []
-    t_start = time.perf_counter()
-    while True:
-        times.append(oracle_round(s1, ow, ost, wl))
-        if max_steps is not None and len(times) >= max_steps:
-            break
-        if time.perf_counter() - t_start > budget or (max_steps is None and sum(times) > 10.0):
-            break
-    t_req = statistics.mean(times)
-    return {"value": s.B / t_req, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
-            "sample": (f"request 0 of {s.C}: its view update (accepted_len new rows), drafter forward "
-                       f"and {s.B}-step correction+sampling in numpy fp64, repeated {len(times)}x "
-                       f"after {warmup} warm-up; round time = {s.C} x sample ({t_req:.2f} s)"),
-            "_t_req": t_req, "_steps": len(times)}
+    while not times or (sum(times) < min_s and sum(times) < budget):
+        times.append(orr.step())
+    t_round = statistics.mean(times)
+    return {"value": s.C * s.B / t_round, "unit": UNIT, "cores": host_cores(), "blas_threads": blas_threads(),
+            "kind": "oracle",
+            "sample": (f"{len(times)} whole round(s) of all {s.C} requests (view update of the round's "
+                       f"new rows, drafter forward, {s.B}-step correction + sampling) in numpy fp64 after "
+                       f"{warmup} warm-up, on the state of a {prefix}-row prefix; mean {t_round:.2f} s per round"),
+            "_t_round": t_round, "_steps": len(times)}
 
 
 # ------------------------------------------------------------------ main
@@ -537,27 +553,119 @@ def workload_config(s, prefix):
 
 
 def run_reference(args, dist, device="cuda"):
-    """The oracle's arm: the same seeded inputs, the oracle alone on the host cores
-    (the library is neither loaded nor run)."""
+    """The oracle's arm: the same seeded inputs and prefix, whole rounds of all C requests
+    by the oracle alone on the host cores (the library is neither loaded nor run):
+    `warmup` untimed rounds, then `steps` timed rounds."""
     if dist.rank != 0:
         return
     s = synth.SHAPES[args.config]
     prefix = args.prefix or s.prefix
     wl = Workload(s, None, synth.input_seed(s) * 1000, device=device)
-    kept = wl.prefix_rows(0, prefix)
-    leg = oracle_leg(wl, kept, args.cpu_budget, max_steps=max(1, args.steps),
-                     warmup=min(args.warmup, 1))
-    ms = leg["_t_req"] * s.C * 1e3
-    out = {"impl": "reference", "metric": METRIC, "value": leg["value"], "unit": UNIT,
-           "n_gpus": args.gpus, "steps": leg["_steps"], "warmup": min(args.warmup, 1),
+    orr = OracleRound(wl, prefix)
+    for _ in range(args.warmup):
+        orr.step()
+    times = [orr.step() for _ in range(max(1, args.steps))]
+    t_round = statistics.mean(times)
+    ms = t_round * 1e3
+    value = s.C * s.B / t_round
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+           "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
            "ms_per_step": ms, "us_per_round": ms * 1e3, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": workload_config(s, prefix),
-           "cpu_baseline": {k: v for k, v in leg.items() if not k.startswith("_")},
-           "e2e": {"value": leg["value"], "unit": UNIT, "h2d_bytes_per_step": 0,
-                   "d2h_bytes_per_step": 0},
-           "note": "steps capped by the time budget; each step is one request's share of a round"}
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "blas_threads": blas_threads(),
+                            "kind": "oracle",
+                            "sample": (f"{len(times)} whole rounds of all {s.C} requests after {args.warmup} "
+                                       f"warm-up, on the state of the {prefix}-row prefix")},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+           "note": "each step is one whole round of all requests by the fp64 oracle on the host cores"}
     print(json.dumps(out), flush=True)
+
+
+def gemm_roofline(s, names, st_ms, hbm, tf_burst, tf_sust, peak_src, traffic_round=None):
+    """The projection GEMM's algorithmic bytes and flops over its stage times."""
+    gemm_bytes = gemm_flops = gemm_ms = 0.0
+    for n, t in zip(names, st_ms):
+        if n in GEMM_STAGES:
+            b, f = gemm_work(s, n)
+            gemm_bytes += b
+            gemm_flops += f
+            gemm_ms += float(t)
+    n_gemm = sum(1 for n in names if n in GEMM_STAGES and (n != "fuse" or not s.no_boundary))
+    ach = gemm_bytes / (gemm_ms * 1e-3) / 1e9
+    intensity = gemm_flops / gemm_bytes
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    return {"bound": "hbm" if intensity < ridge else "tensor",
+            "kernel": f"gemm_kernel (tcgen05 projection GEMM, {n_gemm} launches per round)",
+            "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+            "peak_source": f"{peak_src} HBM copy bandwidth",
+            "traffic": (traffic_round / n_gemm) if traffic_round else None,
+            "algorithmic_bytes_per_launch": gemm_bytes / n_gemm,
+            "avg_launch_us": gemm_ms * 1e3 / n_gemm,
+            "tensor_tflops": tflops,
+            "tensor_frac_of_burst": tflops / tf_burst,
+            "tensor_frac_of_sustained": tflops / tf_sust,
+            "intensity_flop_per_byte": intensity}
+
+
+def round_roofline(s, ms, mean_delta, hbm, tf_burst):
+    rb, rf = round_work(s, mean_delta)
+    t_b, t_f = rb / (hbm * 1e9), rf / (tf_burst * 1e12)
+    t_roof = max(t_b, t_f)
+    return {"bytes": rb, "flops": rf, "bound": "hbm" if t_b >= t_f else "tensor",
+            "roofline_us": t_roof * 1e6, "frac": t_roof * 1e3 / ms}
+
+
+def stage_dict(names, st_ms):
+    stages = {}
+    for n, t in zip(names, st_ms):
+        stages[n] = stages.get(n, 0.0) + float(t) * 1e3
+    return {k: round(v, 2) for k, v in stages.items()}
+
+
+def configs_leg(lsp, dist, hbm, tf_burst, tf_sust, peak_src, steps=200, warmup=10):
+    """The other workload shapes at their own prefixes on the same kernels: the fp32
+    reference shape, the small bf16 shape, and the larger target (C = 32, 128K prefix,
+    the tensor-bound one) sampled at T = 1 and greedy.  Per shape: device time per round
+    (CUDA-graph replay), drafted tokens/s, the round's roofline, and the projection
+    GEMM's HBM and tensor-pipe fractions from the per-stage events."""
+    out = {}
+    legs = (("tiny", "tiny", (None,)), ("small", "small", (None,)), ("large", "large", (1.0, 0.0)))
+    for key, name, temps in legs:
+        s0 = synth.SHAPES[name]
+        wl = Workload(s0, lsp, synth.input_seed(s0) * 1000)
+        st = wl.new_state()
+        wl.fold(st, 0, s0.prefix)
+        for T in temps:
+            s = s0 if T is None else s0.with_(temperature=T)
+            wl.s = s
+            wl.sp = lsp.make_sample_params(s.temperature, seed=synth.RNG_SEED, rnd=0)
+            for _ in range(2):
+                wl.round(st)
+            g = wl.capture(st)
+            ms, _ = time_graph(g, steps, warmup, dist)
+            ms = dist.max(ms)
+            del g
+            names, st_ms = stage_times(wl, st, reps=20)
+            rc, bits = lsp.lsp_get_error(st)
+            if rc != lsp.LSP_OK:
+                raise RuntimeError(f"device error in the {name} leg: {rc} bits={bits}")
+            mean_delta = float(wl.acc.float().mean())
+            leg = {"workload": workload_config(s, s.prefix)["workload"], "C": s.C, "B": s.B,
+                   "prefix": s.prefix, "temperature": s.temperature,
+                   "us_per_round": ms * 1e3, "drafted_tokens_per_s": job_throughput(dist.world, s.C, s.B, ms),
+                   "round_roofline": round_roofline(s, ms, mean_delta, hbm, tf_burst),
+                   "gemm": {k: v for k, v in gemm_roofline(s, names, st_ms, hbm, tf_burst, tf_sust, peak_src).items()
+                            if k in ("bound", "achieved", "frac", "tensor_tflops", "tensor_frac_of_burst",
+                                     "tensor_frac_of_sustained", "avg_launch_us")},
+                   "stages_us": stage_dict(names, st_ms), "launches": lsp.lsp_round_launches(st),
+                   "dtype": s.dtype}
+            out[key if T is None else f"{key}_{'T1' if T > 0 else 'greedy'}"] = leg
+        lsp.lsp_state_destroy(st)
+        del wl
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_ours(args, dist):
@@ -573,8 +681,7 @@ def run_ours(args, dist):
     wl = Workload(s, lsp, synth.input_seed(s) * 1000)
     st = wl.new_state()
     want_cpu = dist.rank == 0 and dist.world == 1 and not args.no_cpu
-    kept = [] if want_cpu else None
-    wl.fold(st, 0, prefix, keep=kept)
+    wl.fold(st, 0, prefix)
     for _ in range(2):
         wl.round(st)
     torch.cuda.synchronize()
@@ -591,35 +698,10 @@ def run_ours(args, dist):
 
     # per-stage device times (dominant kernel = the projection GEMM)
     names, st_ms = stage_times(wl, st, reps=min(200, max(20, args.steps // 5)))
-    gemm_bytes = gemm_flops = gemm_ms = 0.0
-    stages = {}
-    for n, t in zip(names, st_ms):
-        stages[n] = stages.get(n, 0.0) + float(t) * 1e3
-        if n in GEMM_STAGES:
-            b, f = gemm_work(s, n)
-            gemm_bytes += b
-            gemm_flops += f
-            gemm_ms += float(t)
-    n_gemm = sum(1 for n in names if n in GEMM_STAGES)
-    ach = gemm_bytes / (gemm_ms * 1e-3) / 1e9
-    intensity = gemm_flops / gemm_bytes
-    ridge = tf_burst * 1e12 / (hbm * 1e9)
-    traffic_round = profiled_traffic("k_gemm", s.name)
-    roofline = {"bound": "hbm" if intensity < ridge else "tensor",
-                "kernel": f"gemm_kernel (tcgen05 projection GEMM, {n_gemm} launches per round)",
-                "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
-                "peak_source": f"{peak_src} HBM copy bandwidth",
-                "traffic": (traffic_round / n_gemm) if traffic_round else None,
-                "algorithmic_bytes_per_launch": gemm_bytes / n_gemm,
-                "avg_launch_us": gemm_ms * 1e3 / n_gemm,
-                "tensor_tflops": gemm_flops / (gemm_ms * 1e-3) / 1e12,
-                "tensor_frac_of_sustained": gemm_flops / (gemm_ms * 1e-3) / 1e12 / tf_sust,
-                "intensity_flop_per_byte": intensity}
+    roofline = gemm_roofline(s, names, st_ms, hbm, tf_burst, tf_sust, peak_src,
+                             profiled_traffic("k_gemm", s.name))
     mean_delta = float(wl.acc.float().mean())
-    rb, rf = round_work(s, mean_delta)
-    t_roof = max(rb / (hbm * 1e9), rf / (tf_burst * 1e12))
-    round_roof = {"bytes": rb, "flops": rf, "roofline_us": t_roof * 1e6,
-                  "frac": t_roof * 1e3 / ms}
+    round_roof = round_roofline(s, ms, mean_delta, hbm, tf_burst)
 
     # end to end through the C ABI with host buffers (pinned), copies inside the timed region
     hk, hv, hh = wl.k.cpu().pin_memory(), wl.v.cpu().pin_memory(), wl.h.cpu().pin_memory()
@@ -679,9 +761,13 @@ def run_ours(args, dist):
     if not args.no_sweep and s.dtype == "bf16":
         variants = variants_leg(s, lsp, wl.seed_base, dist)
 
+    configs = None
+    if not args.no_sweep and s.name in ("qwen3-8b", "qwen3-8b-sweep"):
+        configs = configs_leg(lsp, dist, hbm, tf_burst, tf_sust, peak_src)
+
     cpu = None
     if want_cpu:
-        leg = oracle_leg(wl, kept, args.cpu_budget)
+        leg = oracle_leg(wl, args.cpu_budget)
         cpu = {k: v for k, v in leg.items() if not k.startswith("_")}
 
     value = job_throughput(dist.world, s.C, s.B, ms)
@@ -692,11 +778,11 @@ def run_ours(args, dist):
            "data": "synthetic (seeded random features and random-init weights)",
            "config": workload_config(s, prefix),
            "roofline": roofline, "round_roofline": round_roof,
-           "stages_us": {k: round(v, 2) for k, v in stages.items()},
+           "stages_us": stage_dict(names, st_ms),
            "e2e": {"value": job_throughput(dist.world, s.C, s.B, e2e_ms), "unit": UNIT,
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
            "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
-           "clocks": clocks, "sweep": sweep, "prefill": prefill, "verify": verify,
+           "clocks": clocks, "sweep": sweep, "configs": configs, "prefill": prefill, "verify": verify,
            "variants": variants, "cpu_baseline": cpu}
     if dist.rank == 0:
         print(json.dumps(out), flush=True)
