@@ -437,7 +437,7 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
   using V = typename std::conditional<EPL == 4, float4, float2>::type;
   float x[EPL];
   {
-    const V v0 = *reinterpret_cast<const V*>(src);
+    const V v0 = __ldcs(reinterpret_cast<const V*>(src));     // partials are read once
     const float* f0 = reinterpret_cast<const float*>(&v0);
 #pragma unroll
     for (int e = 0; e < EPL; ++e) x[e] = f0[e];
@@ -446,7 +446,7 @@ __global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
     V y[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u)
-      if (s0 + u < p.splits) y[u] = *reinterpret_cast<const V*>(src + (size_t)(s0 + u) * pstride);
+      if (s0 + u < p.splits) y[u] = __ldcs(reinterpret_cast<const V*>(src + (size_t)(s0 + u) * pstride));
 #pragma unroll
     for (int u = 0; u < 8; ++u)
       if (s0 + u < p.splits) {

