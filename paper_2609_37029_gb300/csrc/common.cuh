@@ -270,6 +270,24 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   return c;
 }
 
+// ---------------------------------------------------------------- Gumbel noise
+// g = -log(-log u), u = ((x >> 9) + 1/2) 2^-23.  The inner log needs full
+// relative accuracy where u is within 2^-5 of 1 (there -log u is as small as
+// 2^-24 and decides the largest noise values): with w = 1 - u, exact in fp32,
+// it is the Taylor series -log(1 - w) = w + w^2/2 + w^3/3 + ..., cut after
+// w^3 (relative error < w^3 / 4 <= 2^-17).  Elsewhere |log u| >= 2^-5 and the
+// fast log's absolute error (~2^-21) is a relative error below 2^-16; the
+// outer log only needs absolute accuracy.  The drafted tokens are compared
+// with the fp64 definition wherever the top-2 gap exceeds 1e-2.
+__device__ __forceinline__ float gumbel_of(uint32_t x) {
+  const uint32_t k = x >> 9;
+  const float u = ((float)k + 0.5f) * 1.1920928955078125e-07f;          // 2^-23
+  const float w = ((float)(8388607u - k) + 0.5f) * 1.1920928955078125e-07f;   // 1 - u, exact
+  const float series = w * fmaf(w, fmaf(w, 0.333333343f, 0.5f), 1.0f);
+  const float l = w < 0.03125f ? series : -__logf(u);
+  return -__logf(l);
+}
+
 // ---------------------------------------------------------------- warp-level mma.sync helpers
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)

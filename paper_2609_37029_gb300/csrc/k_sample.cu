@@ -45,13 +45,6 @@ constexpr int kMaxC = 64;
 constexpr int kMaxPartialsPerLane = 16;    // sampler grids of up to 512 CTAs
 
 
-// g = -log(-log u): the inner log keeps full relative accuracy (u can be within
-// 2^-24 of 1, where -log u is tiny); the outer log only needs absolute accuracy.
-__device__ __forceinline__ float gumbel_of(uint32_t x) {
-  const float u = ((float)(x >> 9) + 0.5f) * 1.1920928955078125e-07f;   // 2^-23
-  return -__logf(-logf(u));
-}
-
 __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }

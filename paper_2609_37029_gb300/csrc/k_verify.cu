@@ -324,7 +324,7 @@ __global__ void __launch_bounds__(kVerThreads, kDrawCtasPerSm) verify_draw_kerne
       const uint32_t xs[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const float sc = lw[e] - __logf(-logf(ver_uniform(xs[e])));
+        const float sc = lw[e] + gumbel_of(xs[e]);
         if (ver_better(sc, 4 * gi + e, bv, bi)) { bv = sc; bi = 4 * gi + e; }
       }
     }
