@@ -13,9 +13,9 @@
 // One CTA per (request b, tapped layer l, KV head g) covers the nq/nkv query
 // heads sharing that KV head (rep * R queries); the new K/V rows are read from
 // HBM once (16-byte vectors) and only the new rows are touched.
-// view_update_mma_kernel (bf16, d = 128, rep * R in {16, 32, 64}): the
-// statistics are an attention of the summary queries over the new rows, run
-// as mma.sync tiles with an online softmax (below).  view_update_kernel (every
+// view_update_mma_kernel (bf16, d = 128, rep * R a multiple of 16 up to
+// 128): the statistics are an attention of the summary queries over the new
+// rows, run as mma.sync tiles with an online softmax (below).  view_update_kernel (every
 // other shape): rows staged in shared memory as fp32; each warp owns whole
 // queries, lanes split the head dimension, and the dot products and the row
 // max/sum reduce with warp shuffles.
@@ -215,21 +215,33 @@ __global__ void __launch_bounds__(kViewThreads)
 }
 
 // ---------------------------------------------------------------- tensor-core variant
-// bf16 storage, d = 128, Q = rep * R in {16, 32, 64}: the summary update is
-// the attention of the Q summary queries over the new rows, so it runs as
-// mma.sync m16n8k16 tiles.  Warp w owns query tile w % MT (16 queries) and
-// head dims [(w / MT) * 8 * NT, +8 NT): per 16-row key chunk S = G K^T (bf16
-// products are exact, fp32 accumulate), an online softmax in registers, and
-// P V with P split into a bf16 high part and the bf16 remainder (two MMAs:
-// ~16 significant bits of every weight).  The stored (eta, m) stay in the
-// accumulator layout in registers from the first load to the final store.
-constexpr int kVuRows = 64;                // new rows staged per pass
+// bf16 storage, d = 128, Q = rep * R = 16 * MT queries (MT <= 8): the summary
+// update is the attention of the Q summary queries over the new rows, so it
+// runs as mma.sync m16n8k16 tiles.  Warp w owns query tile w (16 queries) and
+// all 128 dims: per 16-row key chunk S = G K^T (bf16 products are exact, fp32
+// accumulate), an online softmax in registers, and P V with P split into a
+// bf16 high part and the bf16 remainder (two MMAs: ~16 significant bits of
+// every weight).  The stored (eta, m) are prefetched into L2 once the
+// dependency wait returns and read only for the final merge, and the G
+// fragments come from shared memory at each k-step, so a CTA needs few
+// registers and 5 CTAs share an SM (Qwen3-8B shape: 640 CTAs in one wave of
+// 760 slots; before, 256-thread CTAs holding the state in registers ran 2.1
+// waves at two per SM).
+constexpr int kVuRows = 32;                // new rows staged per pass
 constexpr int kVuLd = 128 + 8;             // smem row (bf16): conflict-free ldmatrix
 
+// CTAs per SM the launch bounds ask for, at most 8: 96 registers a thread
+// suffice for 4 and 5 query tiles (no spills), the other counts take 112
+constexpr int vu_min_blocks(int MT) {
+  return (MT == 4 || MT == 5) ? 65536 / (MT * 32 * 96)
+                              : (65536 / (MT * 32 * 112) > 8 ? 8 : 65536 / (MT * 32 * 112));
+}
+
 template <int MT>
-__global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const ViewParams p) {
-  constexpr int NT = 16 * MT / kViewWarps;                 // 8-dim output tiles per warp
+__global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_kernel(const ViewParams p) {
+  constexpr int NT = 16;                                   // 8-dim output tiles per warp (all 128 dims)
   constexpr int Q = 16 * MT;
+  constexpr int kThreads = MT * 32;
   extern __shared__ __align__(16) uint8_t vsm_raw[];
   bf16* sG = reinterpret_cast<bf16*>(vsm_raw);             // [Q][kVuLd]
   bf16* sK = sG + Q * kVuLd;                               // [kVuRows][kVuLd]
@@ -241,12 +253,11 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
   const int b = unit / (p.nkv * p.L);
   const int rep = p.nq / p.nkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int mt = warp % MT, d0 = (warp / MT) * 8 * NT;     // this warp's query tile and first dim
   griddep_launch();
   // the summary queries are a constant of the state: stage them before the wait
   const size_t gbase = ((size_t)l * p.nq + (size_t)g * rep) * p.R;
   const bf16* Gp = static_cast<const bf16*>(p.G) + gbase * d;
-  for (int i = tid; i < Q * 16; i += kViewThreads) {
+  for (int i = tid; i < Q * 16; i += kThreads) {
     const int q = i >> 4, c = (i & 15) * 8;
     cp_async16(sG + q * kVuLd + c, Gp + (size_t)q * d + c);
   }
@@ -261,26 +272,11 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
   if (delta == 0) { cp_async_wait_all(); return; }        // empty new set: state unchanged (App. A.2)
   const long long t0 = p.t[b];
 
-  // ---- the stored state of this warp's rows (r0, r0 + 8) and dims, accumulator layout
+  // the stored state of this CTA's Q rows (m: Q x 512 B, eta: Q x 4 B) into L2 for the merge
   const size_t qbase = ((size_t)(b * p.L + l) * p.nq + (size_t)g * rep) * p.R;
-  const int r0 = mt * 16 + (lane >> 2);
-  float* mA = p.m + (qbase + r0) * d + d0 + (lane & 3) * 2;
-  float acc[NT][4];
-#pragma unroll
-  for (int n = 0; n < NT; ++n) {
-    const float2 x0 = *reinterpret_cast<const float2*>(mA + n * 8);
-    const float2 x1 = *reinterpret_cast<const float2*>(mA + 8 * d + n * 8);
-    acc[n][0] = x0.x; acc[n][1] = x0.y; acc[n][2] = x1.x; acc[n][3] = x1.y;
-  }
-  const float etaA0 = p.eta[qbase + r0], etaA1 = p.eta[qbase + r0 + 8];
-  cp_async_wait_all();
-  __syncthreads();
-  // A operand (G rows of this warp's tile) for the 8 k-steps, kept in registers
-  uint32_t ga[8][4];
-  {
-    const bf16* qa = sG + (size_t)(mt * 16 + (lane & 15)) * kVuLd + (lane >> 4) * 8;
-#pragma unroll
-    for (int kk = 0; kk < 8; ++kk) ldsm_x4(ga[kk], qa + kk * 16);
+  if (tid == 0) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.m + qbase * d), "r"((uint32_t)(Q * d * 4))
+                 : "memory");
   }
 
   const float sl2 = 1.4426950408889634f * rsqrtf((float)d);   // log2(e) / sqrt(d)
@@ -296,26 +292,35 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
   const size_t row_stride = (size_t)p.nkv * d;
   const size_t in_base = (size_t)(b * p.L + l) * p.rows * row_stride + (size_t)g * d;
   const size_t win_base = ((size_t)(b * p.L + l) * p.nkv + g) * (size_t)p.W * d;
+  const bf16* qa = sG + (size_t)(warp * 16 + (lane & 15)) * kVuLd + (lane >> 4) * 8;
 
   for (int j0 = 0; j0 < delta; j0 += kVuRows) {
     const int nrows = min(kVuRows, delta - j0);
     const int nrows16 = (nrows + 15) / 16 * 16;
     __syncthreads();                                       // previous rows consumed
-    // stage K and V rows (zero past nrows) and write the window ring
-    for (int idx = tid; idx < 2 * nrows16 * 16; idx += kViewThreads) {
+    // stage K and V rows (zero past nrows) by cp.async: no registers held
+    // across the accumulators
+    for (int idx = tid; idx < 2 * nrows16 * 16; idx += kThreads) {
       const int which = idx / (nrows16 * 16), rem = idx % (nrows16 * 16);
       const int j = rem >> 4, c = (rem & 15) * 8;
-      uint4 raw = make_uint4(0u, 0u, 0u, 0u);
-      if (j < nrows) {
-        raw = *reinterpret_cast<const uint4*>((which ? vin : kin) + in_base + (size_t)(j0 + j) * row_stride + c);
-        if (p.W > 0 && j0 + j >= delta - p.W) {
+      bf16* dst = (which ? sV : sK) + j * kVuLd + c;
+      if (j < nrows) cp_async16(dst, (which ? vin : kin) + in_base + (size_t)(j0 + j) * row_stride + c);
+      else *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    cp_async_wait_all();                                   // (the first pass also lands sG)
+    __syncthreads();
+    // the window ring: the last W rows of the new set, from shared memory
+    if (p.W > 0) {
+      for (int idx = tid; idx < 2 * nrows * 16; idx += kThreads) {
+        const int which = idx / (nrows * 16), rem = idx % (nrows * 16);
+        const int j = rem >> 4, c = (rem & 15) * 8;
+        if (j0 + j >= delta - p.W) {
           const long long pabs = t0 + j0 + j;
-          *reinterpret_cast<uint4*>((which ? wv : wk) + win_base + (size_t)(pabs % p.W) * d + c) = raw;
+          *reinterpret_cast<uint4*>((which ? wv : wk) + win_base + (size_t)(pabs % p.W) * d + c) =
+              *reinterpret_cast<const uint4*>((which ? sV : sK) + j * kVuLd + c);
         }
       }
-      *reinterpret_cast<uint4*>((which ? sV : sK) + j * kVuLd + c) = raw;
     }
-    __syncthreads();
     for (int c16 = 0; c16 < nrows16; c16 += 16) {
       // S = G K^T over 16 keys: two n8 tiles
       float sc[2][4];
@@ -324,10 +329,11 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
       const bf16* kb = sK + (size_t)(c16 + (lane & 7) + (lane >> 4) * 8) * kVuLd + ((lane >> 3) & 1) * 8;
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
-        uint32_t bk[4];
+        uint32_t ga[4], bk[4];
+        ldsm_x4(ga, qa + kk * 16);
         ldsm_x4(bk, kb + kk * 16);
-        mma_bf16(sc[0], ga[kk], bk[0], bk[1]);
-        mma_bf16(sc[1], ga[kk], bk[2], bk[3]);
+        mma_bf16(sc[0], ga, bk[0], bk[1]);
+        mma_bf16(sc[1], ga, bk[2], bk[3]);
       }
       const int nvalid = nrows - c16;
 #pragma unroll
@@ -371,7 +377,7 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
         pl[0] = pack_bf16(rem_of(q00), rem_of(q01)); pl[1] = pack_bf16(rem_of(q02), rem_of(q03));
         pl[2] = pack_bf16(rem_of(q10), rem_of(q11)); pl[3] = pack_bf16(rem_of(q12), rem_of(q13));
       }
-      const bf16* vb = sV + (size_t)(c16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kVuLd + d0 + (lane >> 4) * 8;
+      const bf16* vb = sV + (size_t)(c16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kVuLd + (lane >> 4) * 8;
 #pragma unroll
       for (int np = 0; np < NT / 2; ++np) {
         uint32_t bv[4];
@@ -389,9 +395,11 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
   rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 2);
 
   // ---- (eta_N, m_N) of the new rows, merged into (eta_A, m_A) by Eq. summary-update
+  const int r0 = warp * 16 + (lane >> 2);
+  float* mA = p.m + (qbase + r0) * d + (lane & 3) * 2;
+  const float etaA[2] = {p.eta[qbase + r0], p.eta[qbase + r0 + 8]};
   const float isd = rsqrtf((float)d);
   const float etaN[2] = {rmax[0] * isd + logf(rsum[0]), rmax[1] * isd + logf(rsum[1])};
-  const float etaA[2] = {etaA0, etaA1};
   float ca[2], cn[2], eta[2];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
@@ -401,13 +409,24 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
     cn[h] = __expf(etaN[h] - eta[h]) / rsum[h];            // m_N = o / rsum
   }
 #pragma unroll
-  for (int n = 0; n < NT; ++n) {
-    const float2 y0 = make_float2(ca[0] * acc[n][0] + cn[0] * o[n][0], ca[0] * acc[n][1] + cn[0] * o[n][1]);
-    const float2 y1 = make_float2(ca[1] * acc[n][2] + cn[1] * o[n][2], ca[1] * acc[n][3] + cn[1] * o[n][3]);
-    *reinterpret_cast<float2*>(mA + n * 8) = y0;
-    *reinterpret_cast<float2*>(mA + 8 * d + n * 8) = y1;
+  for (int n0 = 0; n0 < NT; n0 += 4) {                     // four tiles of the stored state in flight
+    float2 x0[4], x1[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      x0[u] = *reinterpret_cast<const float2*>(mA + (n0 + u) * 8);
+      x1[u] = *reinterpret_cast<const float2*>(mA + 8 * d + (n0 + u) * 8);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int n = n0 + u;
+      *reinterpret_cast<float2*>(mA + n * 8) =
+          make_float2(ca[0] * x0[u].x + cn[0] * o[n][0], ca[0] * x0[u].y + cn[0] * o[n][1]);
+      *reinterpret_cast<float2*>(mA + 8 * d + n * 8) =
+          make_float2(ca[1] * x1[u].x + cn[1] * o[n][2], ca[1] * x1[u].y + cn[1] * o[n][3]);
+    }
   }
-  if (d0 == 0 && (lane & 3) == 0) {
+  __syncwarp();                                            // every lane has read eta_A
+  if ((lane & 3) == 0) {
     p.eta[qbase + r0] = eta[0];
     p.eta[qbase + r0 + 8] = eta[1];
   }
@@ -417,7 +436,7 @@ __global__ void __launch_bounds__(kViewThreads, 2) view_update_mma_kernel(const 
     const bf16* hin = static_cast<const bf16*>(p.h_new) + ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
     bf16* hout = static_cast<bf16*>(p.h) + (size_t)(b * p.L + l) * p.H;
     const int per = p.H / p.nkv;
-    for (int i = g * per + tid * 8; i < (g + 1) * per; i += kViewThreads * 8)
+    for (int i = g * per + tid * 8; i < (g + 1) * per; i += kThreads * 8)
       *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
   }
   // ---- the last CTA of request b advances t
@@ -446,7 +465,7 @@ static int launch_mma(const ViewParams& p, cudaStream_t s) {
       return LSP_ERR_CUDA;
     attr = smem;
   }
-  return launch_pdl(view_update_mma_kernel<MT>, dim3(p.C * p.L * p.nkv), dim3(kViewThreads), smem, s, p) ==
+  return launch_pdl(view_update_mma_kernel<MT>, dim3(p.C * p.L * p.nkv), dim3(MT * 32), smem, s, p) ==
                  cudaSuccess
              ? LSP_OK
              : LSP_ERR_CUDA;
@@ -471,12 +490,20 @@ static int launch_dpl(const ViewParams& p, cudaStream_t s) {
 }
 
 int launch_view_update(const ViewParams& p, int dtype, cudaStream_t s) {
-  // tensor-core path: bf16, d = 128, Q = rep * R a power of two from 16 to 64
+  // tensor-core path: bf16, d = 128, Q = rep * R a multiple of 16 up to 128
   const int Q = (p.nq / p.nkv) * p.R;
-  if (dtype == LSP_DTYPE_BF16 && p.d == 128 && view_mma_enabled()) {
-    if (Q == 64) return launch_mma<4>(p, s);
-    if (Q == 32) return launch_mma<2>(p, s);
-    if (Q == 16) return launch_mma<1>(p, s);
+  if (dtype == LSP_DTYPE_BF16 && p.d == 128 && view_mma_enabled() && Q % 16 == 0) {
+    switch (Q / 16) {
+      case 1: return launch_mma<1>(p, s);
+      case 2: return launch_mma<2>(p, s);
+      case 3: return launch_mma<3>(p, s);
+      case 4: return launch_mma<4>(p, s);
+      case 5: return launch_mma<5>(p, s);
+      case 6: return launch_mma<6>(p, s);
+      case 7: return launch_mma<7>(p, s);
+      case 8: return launch_mma<8>(p, s);
+      default: break;
+    }
   }
   if (p.d == 128) return dtype == LSP_DTYPE_BF16 ? launch_dpl<bf16, 4>(p, s) : launch_dpl<float, 4>(p, s);
   if (p.d == 64) return dtype == LSP_DTYPE_BF16 ? launch_dpl<bf16, 2>(p, s) : launch_dpl<float, 2>(p, s);

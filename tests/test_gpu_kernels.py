@@ -91,9 +91,14 @@ def test_linear_matches_fp64_matmul(lsp, M, N, K, dt, splits):
 VU = synth.LspShape("vu", C=3, B=16, L=2, D=1, H=256, nq=8, nkv=2, d=128, F=256, V=1024, W=40,
                     R=16, rc=16)
 VU32 = VU.with_(name="vu32", dtype="f32", nq=4, d=64)
+# rep * R summary queries per KV head: 64 above; the tensor-core kernel takes every
+# multiple of 16 up to 128 (16 x 1..8), the FMA kernel the rest
+VU_Q = {"q16": VU.with_(name="vu16", nq=2), "q48": VU.with_(name="vu48", nq=6),
+        "q80": VU.with_(name="vu80", nq=10), "q128": VU.with_(name="vu128", nq=8, nkv=1),
+        "q24-fma": VU.with_(name="vu24", R=6)}
 
 
-@pytest.mark.parametrize("s", [VU, VU32], ids=["bf16", "f32"])
+@pytest.mark.parametrize("s", [VU, VU32, *VU_Q.values()], ids=["bf16", "f32", *VU_Q])
 def test_view_update_matches_oracle(lsp, s):
     cfg = lsp.make_config(s)
     st = lsp.lsp_state_create(cfg)
