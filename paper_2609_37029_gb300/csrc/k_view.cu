@@ -221,14 +221,27 @@ __global__ void __launch_bounds__(kViewThreads)
 // all 128 dims: per 16-row key chunk S = G K^T (bf16 products are exact, fp32
 // accumulate), an online softmax in registers, and P V with P split into a
 // bf16 high part and the bf16 remainder (two MMAs: ~16 significant bits of
-// every weight).  The stored (eta, m) are prefetched into L2 once the
-// dependency wait returns and read only for the final merge, and the G
-// fragments come from shared memory at each k-step, so a CTA needs few
-// registers and 5 CTAs share an SM (Qwen3-8B shape: 640 CTAs in one wave of
-// 760 slots; before, 256-thread CTAs holding the state in registers ran 2.1
-// waves at two per SM).
+// every weight).  Few registers a thread (the G fragments come from shared
+// memory at each k-step, the stored state is not held), so 5 CTAs share an
+// SM: at the Qwen3-8B shape all 640 CTAs run in one wave of 760 slots.
+//
+// The kernel is a latency chain per CTA (the whole grid moves ~45 MB), so the
+// steps overlap where they can: G is staged before the dependency wait; the
+// stored m block is prefetched into L2 and the boundary row copied while the
+// new K/V rows land; the merge goes through shared memory so that one
+// coalesced pass has all 16 loads a thread in flight at once (instead of four
+// dependent rounds from the MMA fragment layout); and the t advance takes a
+// ticket early instead of a fence after the stores.
 constexpr int kVuRows = 32;                // new rows staged per pass
 constexpr int kVuLd = 128 + 8;             // smem row (bf16): conflict-free ldmatrix
+constexpr int kVuMLd = 128 + 8;            // merge row (fp32): conflict-free float2 stores
+
+// dynamic shared memory: the staging buffers, later reused by the merge
+constexpr size_t vu_smem_bytes(int MT) {
+  const size_t stage = (size_t)(16 * MT + 2 * kVuRows) * kVuLd * 2;
+  const size_t merge = (size_t)16 * MT * (kVuMLd + 1) * 4;
+  return stage > merge ? stage : merge;
+}
 
 // CTAs per SM the launch bounds ask for, at most 8: 96 registers a thread
 // suffice for 4 and 5 query tiles (no spills), the other counts take 112
@@ -261,23 +274,39 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
     const int q = i >> 4, c = (i & 15) * 8;
     cp_async16(sG + q * kVuLd + c, Gp + (size_t)q * d + c);
   }
+  const bf16* kin = static_cast<const bf16*>(p.k_new);
+  const bf16* vin = static_cast<const bf16*>(p.v_new);
+  const size_t row_stride = (size_t)p.nkv * d;
+  const size_t in_base = (size_t)(b * p.L + l) * p.rows * row_stride + (size_t)g * d;
+  // rows [j0, j0 + nv) of the new K and V into sK / sV by cp.async, zeros up to n16
+  auto stage = [&](int j0, int nv, int n16) {
+    for (int idx = tid; idx < 2 * n16 * 16; idx += kThreads) {
+      const int which = idx / (n16 * 16), rem = idx % (n16 * 16);
+      const int j = rem >> 4, c = (rem & 15) * 8;
+      bf16* dst = (which ? sV : sK) + j * kVuLd + c;
+      if (j < nv) cp_async16(dst, (which ? vin : kin) + in_base + (size_t)(j0 + j) * row_stride + c);
+      else *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
   griddep_wait();
-
   const int delta = p.acc[b];
+  const long long t0 = p.t[b];
+  const size_t qbase = ((size_t)(b * p.L + l) * p.nq + (size_t)g * rep) * p.R;
+  const int r0 = warp * 16 + (lane >> 2);
+  const float etaA[2] = {p.eta[qbase + r0], p.eta[qbase + r0 + 8]};
   if (delta < 0 || delta > p.rows) {
     if (tid == 0 && g == 0 && l == 0) set_err(p.err, LSP_DEV_BAD_DELTA);
     cp_async_wait_all();
     return;
   }
   if (delta == 0) { cp_async_wait_all(); return; }        // empty new set: state unchanged (App. A.2)
-  const long long t0 = p.t[b];
-
-  // the stored state of this CTA's Q rows (m: Q x 512 B, eta: Q x 4 B) into L2 for the merge
-  const size_t qbase = ((size_t)(b * p.L + l) * p.nq + (size_t)g * rep) * p.R;
-  if (tid == 0) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.m + qbase * d), "r"((uint32_t)(Q * d * 4))
-                 : "memory");
-  }
+  // t[b] may change once every CTA of request b has read it: each CTA takes a
+  // ticket now (a release atomic, ordered after the read of t) and the CTA that
+  // takes the last one writes t[b] when it is done.  The ticket is consumed
+  // only at the end, so nothing waits on it.
+  int ticket = 0;
+  if (tid == 0)
+    asm volatile("atom.add.release.gpu.global.s32 %0, [%1], 1;" : "=r"(ticket) : "l"(p.done + b) : "memory");
 
   const float sl2 = 1.4426950408889634f * rsqrtf((float)d);   // log2(e) / sqrt(d)
   float rmax[2] = {-INFINITY, -INFINITY}, rsum[2] = {0.f, 0.f};
@@ -285,27 +314,28 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
 #pragma unroll
   for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
 
-  const bf16* kin = static_cast<const bf16*>(p.k_new);
-  const bf16* vin = static_cast<const bf16*>(p.v_new);
   bf16* wk = static_cast<bf16*>(p.win_k);
   bf16* wv = static_cast<bf16*>(p.win_v);
-  const size_t row_stride = (size_t)p.nkv * d;
-  const size_t in_base = (size_t)(b * p.L + l) * p.rows * row_stride + (size_t)g * d;
   const size_t win_base = ((size_t)(b * p.L + l) * p.nkv + g) * (size_t)p.W * d;
   const bf16* qa = sG + (size_t)(warp * 16 + (lane & 15)) * kVuLd + (lane >> 4) * 8;
 
   for (int j0 = 0; j0 < delta; j0 += kVuRows) {
     const int nrows = min(kVuRows, delta - j0);
     const int nrows16 = (nrows + 15) / 16 * 16;
-    __syncthreads();                                       // previous rows consumed
-    // stage K and V rows (zero past nrows) by cp.async: no registers held
-    // across the accumulators
-    for (int idx = tid; idx < 2 * nrows16 * 16; idx += kThreads) {
-      const int which = idx / (nrows16 * 16), rem = idx % (nrows16 * 16);
-      const int j = rem >> 4, c = (rem & 15) * 8;
-      bf16* dst = (which ? sV : sK) + j * kVuLd + c;
-      if (j < nrows) cp_async16(dst, (which ? vin : kin) + in_base + (size_t)(j0 + j) * row_stride + c);
-      else *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    if (j0 > 0) __syncthreads();                           // previous rows consumed
+    stage(j0, nrows, nrows16);
+    if (j0 == 0) {
+      if (tid == 0)                                        // the stored m block into L2 for the merge
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.m + qbase * d), "r"((uint32_t)(Q * d * 4))
+                     : "memory");
+      // boundary: hidden state of the last new row, this CTA's 1/nkv share
+      if (p.h) {
+        const bf16* hin = static_cast<const bf16*>(p.h_new) + ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
+        bf16* hout = static_cast<bf16*>(p.h) + (size_t)(b * p.L + l) * p.H;
+        const int per = p.H / p.nkv;
+        for (int i = g * per + tid * 8; i < (g + 1) * per; i += kThreads * 8)
+          *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
+      }
     }
     cp_async_wait_all();                                   // (the first pass also lands sG)
     __syncthreads();
@@ -395,9 +425,6 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
   rsum[1] += __shfl_xor_sync(0xffffffffu, rsum[1], 2);
 
   // ---- (eta_N, m_N) of the new rows, merged into (eta_A, m_A) by Eq. summary-update
-  const int r0 = warp * 16 + (lane >> 2);
-  float* mA = p.m + (qbase + r0) * d + (lane & 3) * 2;
-  const float etaA[2] = {p.eta[qbase + r0], p.eta[qbase + r0 + 8]};
   const float isd = rsqrtf((float)d);
   const float etaN[2] = {rmax[0] * isd + logf(rsum[0]), rmax[1] * isd + logf(rsum[1])};
   float ca[2], cn[2], eta[2];
@@ -408,47 +435,44 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
     ca[h] = __expf(etaA[h] - eta[h]);
     cn[h] = __expf(etaN[h] - eta[h]) / rsum[h];            // m_N = o / rsum
   }
+  // e^(eta_N - eta) m_N and e^(eta_A - eta) into shared memory (over the
+  // staging buffers, once every warp is done with them) ...
+  float* sM = reinterpret_cast<float*>(vsm_raw);           // [Q][kVuMLd]
+  float* sCa = sM + Q * kVuMLd;                            // [Q]
+  __syncthreads();
 #pragma unroll
-  for (int n0 = 0; n0 < NT; n0 += 4) {                     // four tiles of the stored state in flight
-    float2 x0[4], x1[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      x0[u] = *reinterpret_cast<const float2*>(mA + (n0 + u) * 8);
-      x1[u] = *reinterpret_cast<const float2*>(mA + 8 * d + (n0 + u) * 8);
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int n = n0 + u;
-      *reinterpret_cast<float2*>(mA + n * 8) =
-          make_float2(ca[0] * x0[u].x + cn[0] * o[n][0], ca[0] * x0[u].y + cn[0] * o[n][1]);
-      *reinterpret_cast<float2*>(mA + 8 * d + n * 8) =
-          make_float2(ca[1] * x1[u].x + cn[1] * o[n][2], ca[1] * x1[u].y + cn[1] * o[n][3]);
-    }
+  for (int n = 0; n < NT; ++n) {
+    *reinterpret_cast<float2*>(sM + r0 * kVuMLd + n * 8 + (lane & 3) * 2) = make_float2(cn[0] * o[n][0], cn[0] * o[n][1]);
+    *reinterpret_cast<float2*>(sM + (r0 + 8) * kVuMLd + n * 8 + (lane & 3) * 2) =
+        make_float2(cn[1] * o[n][2], cn[1] * o[n][3]);
   }
-  __syncwarp();                                            // every lane has read eta_A
   if ((lane & 3) == 0) {
-    p.eta[qbase + r0] = eta[0];
+    sCa[r0] = ca[0];
+    sCa[r0 + 8] = ca[1];
+    p.eta[qbase + r0] = eta[0];                            // each eta_A was read above by its own lane
     p.eta[qbase + r0 + 8] = eta[1];
   }
-
-  // ---- boundary: hidden state of the last new row, this CTA's 1/nkv share
-  if (p.h) {
-    const bf16* hin = static_cast<const bf16*>(p.h_new) + ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
-    bf16* hout = static_cast<bf16*>(p.h) + (size_t)(b * p.L + l) * p.H;
-    const int per = p.H / p.nkv;
-    for (int i = g * per + tid * 8; i < (g + 1) * per; i += kThreads * 8)
-      *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);
-  }
-  // ---- the last CTA of request b advances t
   __syncthreads();
-  if (tid == 0) {
+  // ... then one coalesced pass over the CTA's Q x d block of m with every load
+  // in flight at once (16 float4 a thread)
+  constexpr int kPer = Q * d / 4 / kThreads;
+  float4* mrow = reinterpret_cast<float4*>(p.m + qbase * d);
+  float4 xa[kPer];
+#pragma unroll
+  for (int u = 0; u < kPer; ++u) xa[u] = mrow[tid + u * kThreads];
+#pragma unroll
+  for (int u = 0; u < kPer; ++u) {
+    const int i = tid + u * kThreads, q = i >> 5, c = (i & 31) * 4;
+    const float a = sCa[q];
+    const float4 nv = *reinterpret_cast<const float4*>(sM + q * kVuMLd + c);
+    mrow[i] = make_float4(a * xa[u].x + nv.x, a * xa[u].y + nv.y, a * xa[u].z + nv.z, a * xa[u].w + nv.w);
+  }
+
+  // ---- the CTA with the last ticket of request b advances t
+  if (tid == 0 && ticket == p.L * p.nkv - 1) {
     __threadfence();
-    const int old = atomicAdd(&p.done[b], 1);
-    if (old == p.L * p.nkv - 1) {
-      p.t[b] = t0 + delta;
-      p.done[b] = 0;
-      __threadfence();
-    }
+    p.t[b] = t0 + delta;
+    p.done[b] = 0;
   }
 }
 
@@ -457,7 +481,7 @@ static bool view_mma_enabled() { return std::getenv("LSP_VIEW_FMA") == nullptr; 
 
 template <int MT>
 static int launch_mma(const ViewParams& p, cudaStream_t s) {
-  const size_t smem = (size_t)(16 * MT + 2 * kVuRows) * kVuLd * sizeof(bf16);
+  const size_t smem = vu_smem_bytes(MT);
   static size_t attr = 0;
   if (smem > attr) {
     if (cudaFuncSetAttribute(view_update_mma_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
