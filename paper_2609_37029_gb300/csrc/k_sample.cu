@@ -354,6 +354,8 @@ __device__ __forceinline__ void gather_e(const bf16* Ec, int y, int C, int rc, u
 }
 
 // KS = rc / 16 k-steps of the m16n8k16 contraction.
+// (17 warps of 32 threads: at 120 registers a thread the occupancy query
+// reports no resident CTA, so the bound stays at 96 registers)
 template <int KS>
 __global__ void __launch_bounds__(kPThreads, 1)
     sample_persistent_kernel(const SampleParams p, const int ntiles) {
@@ -404,45 +406,34 @@ __global__ void __launch_bounds__(kPThreads, 1)
     }
   }
 
-  auto issue_z = [&](int s) {        // this lane's own logits of step s (same lane reads them)
+  // this lane's own logits of step s for local tile lt (the same lane reads them)
+  auto issue_z_tile = [&](int s, int lt) {
+    const int v = (t_begin + lt) * 16 + 4 * q;
 #pragma unroll
-    for (int j = 0; j < kPTilesPerWarp; ++j) {
-      const int lt = warp + kPWarps * j;
-      if (lt < cnt) {
-        const int v = (t_begin + lt) * 16 + 4 * q;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int r = g + 8 * h;
-          const bool ok = r < C;
-          cp_async16(&Zs[(lt * 2 + h) * 32 + lane], p.src + (ok ? ((size_t)r * B + s) * V + v : 0),
-                     ok ? 16u : 0u);
-        }
-      }
+    for (int h = 0; h < 2; ++h) {
+      const int r = g + 8 * h;
+      const bool ok = r < C;
+      cp_async16(&Zs[(lt * 2 + h) * 32 + lane], p.src + (ok ? ((size_t)r * B + s) * V + v : 0), ok ? 16u : 0u);
     }
   };
   float gn[kPTilesPerWarp][2][4];      // noise of the step about to be scored
-  auto draw_noise = [&](int s) {
+  auto draw_noise_tile = [&](int s, int j, int lt) {
+    const int v = (t_begin + lt) * 16 + 4 * q;
 #pragma unroll
-    for (int j = 0; j < kPTilesPerWarp; ++j) {
-      const int lt = warp + kPWarps * j;
-      if (lt < cnt) {
-        const int v = (t_begin + lt) * 16 + 4 * q;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const uint4 x = philox4x32_10(
-              make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(g + 8 * h), p.round), key);
-          gn[j][h][0] = gumbel_of(x.x);
-          gn[j][h][1] = gumbel_of(x.y);
-          gn[j][h][2] = gumbel_of(x.z);
-          gn[j][h][3] = gumbel_of(x.w);
-        }
-      }
+    for (int h = 0; h < 2; ++h) {
+      const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(g + 8 * h), p.round), key);
+      gn[j][h][0] = gumbel_of(x.x);
+      gn[j][h][1] = gumbel_of(x.y);
+      gn[j][h][2] = gumbel_of(x.z);
+      gn[j][h][3] = gumbel_of(x.w);
     }
   };
 
   int y = 0;                                                            // control warp: y of lane < C
   if (warp < kPWarps) {
-    issue_z(0);
+#pragma unroll
+    for (int j = 0; j < kPTilesPerWarp; ++j)
+      if (warp + kPWarps * j < cnt) issue_z_tile(0, warp + kPWarps * j);
   } else {
     __syncwarp();
     if (lane < C) {
@@ -456,7 +447,11 @@ __global__ void __launch_bounds__(kPThreads, 1)
   asm volatile("cp.async.commit_group;" ::: "memory");
   __syncthreads();                                                      // E rows zeroed
   if (warp == kPWarps) gather_e<CH>(Ec, y, C, rc, Es, lane);
-  if (warp < kPWarps && sample) draw_noise(0);
+  if (warp < kPWarps && sample) {
+#pragma unroll
+    for (int j = 0; j < kPTilesPerWarp; ++j)
+      if (warp + kPWarps * j < cnt) draw_noise_tile(0, j, warp + kPWarps * j);
+  }
   asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();                                                      // W_c slice and E_c(y_0) visible
 
@@ -532,12 +527,15 @@ __global__ void __launch_bounds__(kPThreads, 1)
       }
       named_arrive(kBarKeys, kPThreads);
       // HBM traffic of this lane (corrected logits out, next logits in) and the
-      // next step's noise overlap the grid-wide wait
-      if (p.dst) {
+      // next step's noise overlap the grid-wide wait; tile by tile, so that the
+      // noise arithmetic of a tile runs while its memory operations drain
+      // instead of the warp stalling on a full store queue
+      const bool more = s + 1 < B;
 #pragma unroll
-        for (int j = 0; j < kPTilesPerWarp; ++j) {
-          const int lt = warp + kPWarps * j;
-          if (lt < cnt) {
+      for (int j = 0; j < kPTilesPerWarp; ++j) {
+        const int lt = warp + kPWarps * j;
+        if (lt < cnt) {
+          if (p.dst) {
             const int v = (t_begin + lt) * 16 + 4 * q;
 #pragma unroll
             for (int h = 0; h < 2; ++h)
@@ -545,12 +543,14 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 *reinterpret_cast<float4*>(p.dst + ((size_t)(g + 8 * h) * B + s) * V + v) =
                     Zs[(lt * 2 + h) * 32 + lane];
           }
+          if (more) {
+            issue_z_tile(s + 1, lt);                                    // slot already consumed
+            if (sample) draw_noise_tile(s + 1, j, lt);
+          }
         }
       }
-      if (s + 1 == B) break;
-      issue_z(s + 1);                                                   // slots already consumed
+      if (!more) break;
       asm volatile("cp.async.commit_group;" ::: "memory");
-      if (sample) draw_noise(s + 1);
       named_bar(kBarNext, kPThreads);
       if (*abort_flag) break;
     }
