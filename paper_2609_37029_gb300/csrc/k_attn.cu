@@ -25,6 +25,7 @@
 // shared memory 64 at a time (float4 loads, several in flight per thread), a
 // warp scores each staged key against all block queries (lanes split over
 // queries and head dims), one softmax, then P V over the re-staged values.
+#include <algorithm>
 #include <type_traits>
 
 #include "common.cuh"
@@ -483,74 +484,98 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
 }
 
 // ------------------------------------------------------------ q/k/v finalisation
-// One warp per (block row, head): the sum of the q/k/v projection's split-K
-// partials in split order, then for q and k heads the per-head RMSNorm and the
-// rotary embedding (pairs f, f + d/2; lane l holds elements EPL*l .. EPL*l+EPL-1,
-// its rotary partner lives in lane l ^ 16).
+// One warp per group of kFinRows (block row, head) rows: the sum of the q/k/v
+// projection's split-K partials in split order, then for q and k heads the
+// per-head RMSNorm and the rotary embedding (pairs f, f + d/2; lane l holds
+// elements EPL*l .. EPL*l+EPL-1, its rotary partner lives in lane l ^ 16).
+// The grid is capped at two CTAs per SM (a grid-stride loop covers the rest),
+// so every CTA is resident as soon as the projection's CTAs leave: the
+// attention kernel, which launches once every CTA here has passed its wait,
+// then starts staging its window while these rows are still being formed.
+// Measured at the Qwen3-8B round with one row per warp (1536 CTAs, 1.4 waves):
+// the attention started ~8.5 us after the projection ended.
+constexpr int kFinRows = 6;
+
 template <typename T, int EPL>
-__global__ void __launch_bounds__(256) qkv_finalize_kernel(const QkvParams p) {
+__global__ void __launch_bounds__(256, 2) qkv_finalize_kernel(const QkvParams p) {
   // wait first, then let the attention kernel launch: it reads the view
   // state before its own wait, which is safe once the q/k/v projection (and
   // so every kernel before it) has completed
   griddep_wait();
   griddep_launch();
   const int heads = p.nq + 2 * p.nkv;
-  const int item = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int items = p.M * heads;
   const int lane = threadIdx.x & 31;
-  if (item >= p.M * heads) return;
-  const int m = item / heads, h = item % heads;
   const int d = EPL * 32, half = d / 2;
   const size_t ldq = (size_t)heads * d;
   const size_t pstride = (size_t)p.M * ldq;
-  const float* src = p.part + (size_t)m * ldq + (size_t)h * d + EPL * lane;
-  // the lane's EPL consecutive values of every split as one vector load each,
-  // all in flight before the adds (which run in split order)
   using V = typename std::conditional<EPL == 4, float4, float2>::type;
-  float x[EPL];
-  {
-    const V v0 = __ldcs(reinterpret_cast<const V*>(src));     // partials are read once
-    const float* f0 = reinterpret_cast<const float*>(&v0);
+  const int nw = gridDim.x * 8;
+  for (int base = (blockIdx.x * 8 + (threadIdx.x >> 5)) * kFinRows; base < items; base += nw * kFinRows) {
+    // kFinRows rows x up to three splits of vector loads in flight before the
+    // adds (which run in split order); partials are read once
+    float x[kFinRows][EPL];
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) x[e] = f0[e];
-  }
-  for (int s0 = 1; s0 < p.splits; s0 += 8) {
-    V y[8];
+    for (int u = 0; u < kFinRows; ++u)
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (s0 + u < p.splits) y[u] = __ldcs(reinterpret_cast<const V*>(src + (size_t)(s0 + u) * pstride));
+      for (int e = 0; e < EPL; ++e) x[u][e] = 0.f;
+    const float* src0 = p.part + (size_t)base * d + EPL * lane;   // rows base.. are contiguous
+    for (int s0 = 0; s0 < p.splits; s0 += 3) {
+      V y[3][kFinRows];
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (s0 + u < p.splits) {
-        const float* f = reinterpret_cast<const float*>(&y[u]);
+      for (int v = 0; v < 3; ++v) {
+        const float* sv = src0 + (size_t)(s0 + v) * pstride;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) x[e] += f[e];
+        for (int u = 0; u < kFinRows; ++u)
+          if (s0 + v < p.splits && base + u < items) y[v][u] = __ldcs(reinterpret_cast<const V*>(sv + u * d));
       }
-  }
-  if (h < p.nq + p.nkv) {
-    const T* w = static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane;
-    float ss = 0.f;
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) ss += x[e] * x[e];
-    const float rstd = rsqrtf(warp_sum(ss) / (float)d + p.eps);
+      for (int v = 0; v < 3; ++v)
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) x[e] *= rstd * to_f(w[e]);
-    const int b = m / p.B, i = m % p.B;
-    const float* cs = p.rope + ((size_t)(b * p.B + i) * half + EPL * (lane & 15)) * 2;
-    const float sg = lane < 16 ? -1.f : 1.f;
+        for (int u = 0; u < kFinRows; ++u)
+          if (s0 + v < p.splits && base + u < items) {
+            const float* f = reinterpret_cast<const float*>(&y[v][u]);
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-      const float partner = __shfl_xor_sync(0xffffffffu, x[e], 16);
-      x[e] = x[e] * cs[2 * e] + sg * partner * cs[2 * e + 1];
+            for (int e = 0; e < EPL; ++e) x[u][e] += f[e];
+          }
+    }
+#pragma unroll
+    for (int u = 0; u < kFinRows; ++u) {
+      const int item = base + u;
+      if (item >= items) break;                      // warp-uniform
+      const int m = item / heads, h = item % heads;
+      if (h < p.nq + p.nkv) {
+        const T* w = static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane;
+        float ss = 0.f;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) ss += x[u][e] * x[u][e];
+        const float rstd = rsqrtf(warp_sum(ss) / (float)d + p.eps);
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) x[u][e] *= rstd * to_f(w[e]);
+        const int b = m / p.B, i = m % p.B;
+        const float* cs = p.rope + ((size_t)(b * p.B + i) * half + EPL * (lane & 15)) * 2;
+        const float sg = lane < 16 ? -1.f : 1.f;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) {
+          const float partner = __shfl_xor_sync(0xffffffffu, x[u][e], 16);
+          x[u][e] = x[u][e] * cs[2 * e] + sg * partner * cs[2 * e + 1];
+        }
+      }
+      T* out = static_cast<T*>(p.out) + (size_t)item * d + EPL * lane;
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) out[e] = from_f<T>(x[u][e]);
     }
   }
-  T* out = static_cast<T*>(p.out) + (size_t)m * ldq + (size_t)h * d + EPL * lane;
-#pragma unroll
-  for (int e = 0; e < EPL; ++e) out[e] = from_f<T>(x[e]);
 }
 
 int launch_qkv_finalize(const QkvParams& p, int dtype, cudaStream_t s) {
   const int items = p.M * (p.nq + 2 * p.nkv);
-  const dim3 grid((items + 7) / 8);
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return LSP_ERR_CUDA;
+  const int need = (items + 8 * kFinRows - 1) / (8 * kFinRows);
+  const dim3 grid(std::min(need, 2 * sms));
   cudaError_t e;
   if (p.d == 128)
     e = dtype == LSP_DTYPE_BF16 ? launch_pdl(qkv_finalize_kernel<bf16, 4>, grid, dim3(256), 0, s, p)
