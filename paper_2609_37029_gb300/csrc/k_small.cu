@@ -143,13 +143,14 @@ __global__ void __launch_bounds__(kRowThreads) combine_kernel(const CombineParam
   }
 }
 
-// One CTA per token row with (up to) one 16-byte vector per thread: every
-// partial load of a thread is in flight at once and 32 warps per row keep the
-// SM busy while they land.
-constexpr int kNormThreads = 1024;
+// One CTA of up to 512 threads per token row (two 16-byte vectors a thread
+// at H = 4096): every partial load of a thread is in flight at once, and an SM
+// keeps room (threads and registers) for a CTA of the projection launched
+// after this kernel, which then starts its weight stream while the norm runs.
+constexpr int kNormThreads = 512;
 
 template <typename T, int VPT>
-__global__ void __launch_bounds__(kNormThreads)
+__global__ void __launch_bounds__(kNormThreads, 2)
     resid_norm_kernel(float* __restrict__ x, const float* __restrict__ part, int splits,
                       const T* __restrict__ w, T* __restrict__ out, int M, int H, float eps) {
   __shared__ float red[32];
@@ -174,20 +175,23 @@ __global__ void __launch_bounds__(kNormThreads)
     const int j = threadIdx.x + k * blockDim.x;
     if (j < h4) xv[k] = ld4(row, j);
   }
-  // splits in groups of eight with all loads issued before the adds (in split order)
-  for (int s0 = 0; s0 < splits; s0 += 8) {
+  // splits in groups with all loads of a group issued before the adds (in split order)
+  constexpr int kGrp = VPT <= 1 ? 8 : VPT == 2 ? 4 : 2;
+  for (int s0 = 0; s0 < splits; s0 += kGrp) {
+    float4 t[VPT][kGrp];
 #pragma unroll
     for (int k = 0; k < VPT; ++k) {
       const int j = threadIdx.x + k * blockDim.x;
-      if (j < h4) {
-        float4 t[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (s0 + u < splits) t[u] = ld4_last(prow + (s0 + u) * pstride, j);
+      for (int u = 0; u < kGrp; ++u)
+        if (j < h4 && s0 + u < splits) t[k][u] = ld4_last(prow + (s0 + u) * pstride, j);
+    }
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (s0 + u < splits) xv[k] = add4(xv[k], t[u]);
-      }
+    for (int k = 0; k < VPT; ++k) {
+      const int j = threadIdx.x + k * blockDim.x;
+#pragma unroll
+      for (int u = 0; u < kGrp; ++u)
+        if (j < h4 && s0 + u < splits) xv[k] = add4(xv[k], t[k][u]);
     }
   }
 #pragma unroll
@@ -228,13 +232,15 @@ static cudaError_t launch_norm_t(float* x, const float* part, int splits, const 
   switch (vpt) {
     case 1: return launch_pdl(resid_norm_kernel<T, 1>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
     case 2: return launch_pdl(resid_norm_kernel<T, 2>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
+    case 3: return launch_pdl(resid_norm_kernel<T, 3>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
+    case 4: return launch_pdl(resid_norm_kernel<T, 4>, dim3(M), dim3(threads), 0, s, x, part, splits, wt, ot, M, H, eps);
     default: return cudaErrorInvalidValue;
   }
 }
 
 int launch_resid_norm(float* x, const float* part, int splits, const void* w, void* out, int M,
                       int H, float eps, int dtype, cudaStream_t s) {
-  if (H > 2 * 4 * kNormThreads || H % 4) return LSP_ERR_SHAPE;
+  if (H > 4 * 4 * kNormThreads || H % 4) return LSP_ERR_SHAPE;
   const cudaError_t e = dtype == LSP_DTYPE_BF16
                             ? launch_norm_t<bf16>(x, part, splits, w, out, M, H, eps, s)
                             : launch_norm_t<float>(x, part, splits, w, out, M, H, eps, s);
