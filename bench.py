@@ -52,6 +52,9 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=150.0, help="seconds for the oracle legs")
+    ap.add_argument("--profile-rounds", type=int, default=0,
+                    help="only fold the prefix and run this many eager rounds, then exit "
+                         "(a short, untimed command for a profiler)")
     return ap.parse_args()
 
 
@@ -789,8 +792,31 @@ def run_ours(args, dist):
     lsp.lsp_state_destroy(st)
 
 
+def profile_rounds(args):
+    """Fold the prefix, run `--profile-rounds` eager rounds, check the device error
+    word and exit: the launch sequence of a round without the timing legs."""
+    from paper_2609_37029_gb300 import build as _b
+    _b.build()
+    from paper_2609_37029_gb300 import lsp
+    s = synth.SHAPES[args.config]
+    wl = Workload(s, lsp, synth.input_seed(s) * 1000)
+    st = wl.new_state()
+    wl.fold(st, 0, args.prefix or s.prefix)
+    for _ in range(args.profile_rounds):
+        wl.round(st)
+    torch.cuda.synchronize()
+    rc, bits = lsp.lsp_get_error(st)
+    lsp.lsp_state_destroy(st)
+    if rc != lsp.LSP_OK:
+        raise RuntimeError(f"device error: {rc} bits={bits}")
+    print(f"{args.profile_rounds} round(s) of {s.name} after a {args.prefix or s.prefix}-row prefix: ok")
+
+
 def main():
     args = parse_args()
+    if args.profile_rounds > 0:
+        profile_rounds(args)
+        return
     dist = Dist()
     try:
         if args.impl == "reference":
