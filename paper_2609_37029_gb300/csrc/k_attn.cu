@@ -484,6 +484,41 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
 }
 
 // ------------------------------------------------------------ q/k/v finalisation
+// N (2 or 4) consecutive fp32 / bf16 values <-> fp32 registers, one vector access
+template <int N>
+__device__ __forceinline__ void load_vec(const float* p, float* v) {
+  if constexpr (N == 4) {
+    const float4 x = *reinterpret_cast<const float4*>(p);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+  } else {
+    const float2 x = *reinterpret_cast<const float2*>(p);
+    v[0] = x.x; v[1] = x.y;
+  }
+}
+template <int N>
+__device__ __forceinline__ void load_vec(const bf16* p, float* v) {
+  if constexpr (N == 4) {
+    const uint2 r = *reinterpret_cast<const uint2*>(p);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
+    v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+  } else {
+    const __nv_bfloat162 r = *reinterpret_cast<const __nv_bfloat162*>(p);
+    const float2 a = __bfloat1622float2(r);
+    v[0] = a.x; v[1] = a.y;
+  }
+}
+template <int N>
+__device__ __forceinline__ void store_vec(float* p, const float* v) {
+  if constexpr (N == 4) *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  else *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+}
+template <int N>
+__device__ __forceinline__ void store_vec(bf16* p, const float* v) {
+  if constexpr (N == 4) *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+  else *reinterpret_cast<uint32_t*>(p) = pack_bf16(v[0], v[1]);
+}
+
 // One warp per group of kFinRows (block row, head) rows: the sum of the q/k/v
 // projection's split-K partials in split order, then for q and k heads the
 // per-head RMSNorm and the rotary embedding (pairs f, f + d/2; lane l holds
@@ -545,15 +580,19 @@ __global__ void __launch_bounds__(256, 2) qkv_finalize_kernel(const QkvParams p)
       if (item >= items) break;                      // warp-uniform
       const int m = item / heads, h = item % heads;
       if (h < p.nq + p.nkv) {
-        const T* w = static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane;
+        // the lane's norm weights and (cos, sin) pairs as vector loads, issued before the reduction
+        float w[EPL], cs[2 * EPL];
+        load_vec<EPL>(static_cast<const T*>(h < p.nq ? p.q_norm : p.k_norm) + EPL * lane, w);
+        const int b = m / p.B, i = m % p.B;
+        const float* csp = p.rope + ((size_t)(b * p.B + i) * half + EPL * (lane & 15)) * 2;
+        load_vec<EPL>(csp, cs);
+        load_vec<EPL>(csp + EPL, cs + EPL);
         float ss = 0.f;
 #pragma unroll
         for (int e = 0; e < EPL; ++e) ss += x[u][e] * x[u][e];
         const float rstd = rsqrtf(warp_sum(ss) / (float)d + p.eps);
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) x[u][e] *= rstd * to_f(w[e]);
-        const int b = m / p.B, i = m % p.B;
-        const float* cs = p.rope + ((size_t)(b * p.B + i) * half + EPL * (lane & 15)) * 2;
+        for (int e = 0; e < EPL; ++e) x[u][e] *= rstd * w[e];
         const float sg = lane < 16 ? -1.f : 1.f;
 #pragma unroll
         for (int e = 0; e < EPL; ++e) {
@@ -561,9 +600,7 @@ __global__ void __launch_bounds__(256, 2) qkv_finalize_kernel(const QkvParams p)
           x[u][e] = x[u][e] * cs[2 * e] + sg * partner * cs[2 * e + 1];
         }
       }
-      T* out = static_cast<T*>(p.out) + (size_t)item * d + EPL * lane;
-#pragma unroll
-      for (int e = 0; e < EPL; ++e) out[e] = from_f<T>(x[u][e]);
+      store_vec<EPL>(static_cast<T*>(p.out) + (size_t)item * d + EPL * lane, x[u]);
     }
   }
 }
