@@ -117,12 +117,19 @@ typedef struct lsp_config {
  *   h[b][l][j][0..H)           hidden state at that row (only row accepted_len-1 is read)
  * All three are device pointers of dtype with row capacity `rows` per (b, l);
  * h may be null (and is not read) with LSP_NO_BOUNDARY.
+ * h_rows: rows of h per (b, l).  0 (the default when the struct is zeroed) or
+ * `rows`: the layout above.  1: h[b][l][0..H) holds only the boundary row --
+ * the hidden state at row accepted_len[b]-1 (for lsp_prefill: at row t-1) --
+ * which is all the interface reads (Sec. 2.2), so a caller that stages the
+ * rows from host memory copies C*L*H elements instead of C*L*rows*H.  Any
+ * other value is LSP_ERR_ARG.
  */
 typedef struct lsp_target_feats {
   const void* k;
   const void* v;
   const void* h;
   int rows;
+  int h_rows;
 } lsp_target_feats;
 
 /* One Qwen3-style draft layer (App. B.1); device pointers of dtype. */

@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(256) prefill_merge_kernel(const PrefillParams 
   }
   if (g == 0) {
     if (p.h) {   // no boundary state is kept with LSP_NO_BOUNDARY
-      const T* hin = static_cast<const T*>(p.hid) + ((size_t)l * p.rows + (p.rows - 1)) * p.H;
+      const T* hin = static_cast<const T*>(p.hid) + ((size_t)l * p.h_rows + (p.h_rows - 1)) * p.H;
       T* hout = static_cast<T*>(p.h) + ((size_t)b * p.L + l) * p.H;
       for (int i = threadIdx.x * vec; i < p.H; i += blockDim.x * vec)
         *reinterpret_cast<uint4*>(hout + i) = *reinterpret_cast<const uint4*>(hin + i);

@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(kViewThreads)
   // ---- boundary: hidden state of the last new row, this CTA's 1/nkv share
   if (p.h) {   // no boundary state is kept with LSP_NO_BOUNDARY
     const T* hin = static_cast<const T*>(p.h_new) +
-                   ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
+                   ((size_t)(b * p.L + l) * p.h_rows + (p.h_rows == 1 ? 0 : delta - 1)) * p.H;
     T* hout = static_cast<T*>(p.h) + (size_t)(b * p.L + l) * p.H;
     const int per = p.H / p.nkv;
     for (int i = g * per + threadIdx.x * vec; i < (g + 1) * per; i += kViewThreads * vec)
@@ -330,7 +330,8 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
                      : "memory");
       // boundary: hidden state of the last new row, this CTA's 1/nkv share
       if (p.h) {
-        const bf16* hin = static_cast<const bf16*>(p.h_new) + ((size_t)(b * p.L + l) * p.rows + (delta - 1)) * p.H;
+        const bf16* hin = static_cast<const bf16*>(p.h_new) +
+                          ((size_t)(b * p.L + l) * p.h_rows + (p.h_rows == 1 ? 0 : delta - 1)) * p.H;
         bf16* hout = static_cast<bf16*>(p.h) + (size_t)(b * p.L + l) * p.H;
         const int per = p.H / p.nkv;
         for (int i = g * per + tid * 8; i < (g + 1) * per; i += kThreads * 8)

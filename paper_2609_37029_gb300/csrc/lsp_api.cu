@@ -307,14 +307,20 @@ int lsp_state_init(lsp_state* st, const void* G, lsp_stream_t stream) {
   return LSP_OK;
 }
 
+// rows of h per (b, l) that a feature struct describes (-1: invalid)
+static int feats_h_rows(const lsp_target_feats* f) {
+  if (f->h_rows == 0 || f->h_rows == f->rows) return f->rows;
+  return f->h_rows == 1 ? 1 : -1;
+}
+
 int lsp_view_update(lsp_state* st, const lsp_target_feats* f, const int32_t* acc,
                     lsp_stream_t stream) {
-  if (!st || !f || !acc || !f->k || !f->v || f->rows < 1) return LSP_ERR_ARG;
+  if (!st || !f || !acc || !f->k || !f->v || f->rows < 1 || feats_h_rows(f) < 0) return LSP_ERR_ARG;
   if (!f->h && st->h) return LSP_ERR_ARG;
   if (!st->initialized) return LSP_ERR_STATE;
   const lsp_config& c = st->cfg;
   ViewParams p;
-  p.k_new = f->k; p.v_new = f->v; p.h_new = f->h; p.rows = f->rows; p.acc = acc;
+  p.k_new = f->k; p.v_new = f->v; p.h_new = f->h; p.rows = f->rows; p.h_rows = feats_h_rows(f); p.acc = acc;
   p.G = st->G; p.win_k = st->win_k; p.win_v = st->win_v; p.m = st->m; p.eta = st->eta;
   p.h = st->h; p.t = st->t; p.done = st->done; p.err = st->err;
   p.C = c.C; p.L = c.L; p.nq = c.nq; p.nkv = c.nkv; p.d = c.d; p.H = c.H; p.W = c.W; p.R = c.R;
@@ -325,13 +331,13 @@ int lsp_view_update(lsp_state* st, const lsp_target_feats* f, const int32_t* acc
 }
 
 int lsp_prefill(lsp_state* st, int b, const lsp_target_feats* f, lsp_stream_t stream) {
-  if (!st || !f || !f->k || !f->v || f->rows < 1) return LSP_ERR_ARG;
+  if (!st || !f || !f->k || !f->v || f->rows < 1 || feats_h_rows(f) < 0) return LSP_ERR_ARG;
   if (!f->h && st->h) return LSP_ERR_ARG;
   if (!st->initialized) return LSP_ERR_STATE;
   const lsp_config& c = st->cfg;
   if (b < 0 || b >= c.C) return LSP_ERR_ARG;
   PrefillParams p;
-  p.k = f->k; p.v = f->v; p.hid = f->h; p.rows = f->rows; p.G = st->G;
+  p.k = f->k; p.v = f->v; p.hid = f->h; p.rows = f->rows; p.h_rows = feats_h_rows(f); p.G = st->G;
   p.win_k = st->win_k; p.win_v = st->win_v; p.m = st->m; p.eta = st->eta; p.h = st->h; p.t = st->t;
   p.ws = st->prefill_ws;
   p.b = b; p.L = c.L; p.nq = c.nq; p.nkv = c.nkv; p.d = c.d; p.W = c.W; p.R = c.R; p.H = c.H;

@@ -97,6 +97,7 @@ struct ViewParams {
   const void* v_new;
   const void* h_new;
   int rows;
+  int h_rows;             // rows of h_new per (b, l): rows, or 1 = only the boundary row
   const int32_t* acc;
   const void* G;
   void* win_k;
@@ -166,8 +167,9 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s);
 struct PrefillParams {
   const void* k;          // request b's prefix K: [L][rows][nkv][d] dtype
   const void* v;          // V, same layout
-  const void* hid;        // hidden states [L][rows][H] dtype
+  const void* hid;        // hidden states [L][h_rows][H] dtype (h_rows = rows or 1: the last row only)
   int rows;               // t (>= 1)
+  int h_rows;
   const void* G;          // [L][nq][R][d]
   void* win_k;            // state window [C][L][nkv][W][d]
   void* win_v;

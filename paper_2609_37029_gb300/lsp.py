@@ -36,7 +36,7 @@ class lsp_config(Structure):
 
 
 class lsp_target_feats(Structure):
-    _fields_ = [("k", c_void_p), ("v", c_void_p), ("h", c_void_p), ("rows", c_int)]
+    _fields_ = [("k", c_void_p), ("v", c_void_p), ("h", c_void_p), ("rows", c_int), ("h_rows", c_int)]
 
 
 _LAYER_FIELDS = ["in_norm", "wq", "wk", "wv", "q_norm", "k_norm", "wo", "post_norm", "w_gate",
@@ -185,15 +185,18 @@ def lsp_state_init(st, G, stream=None) -> None:
     _check(_f["lsp_state_init"](st, _ptr(G), _stream(stream)), "lsp_state_init")
 
 
-def lsp_view_update(st, k, v, h, accepted_len, rows=None, stream=None) -> None:
-    f = lsp_target_feats(_ptr(k), _ptr(v), _ptr(h), int(rows if rows is not None else k.shape[2]))
+def lsp_view_update(st, k, v, h, accepted_len, rows=None, stream=None, h_rows=0) -> None:
+    """h_rows = 1: h is [C][L][1][H], the hidden state of each request's last new row only."""
+    f = lsp_target_feats(_ptr(k), _ptr(v), _ptr(h), int(rows if rows is not None else k.shape[2]), int(h_rows))
     _check(_f["lsp_view_update"](st, ctypes.byref(f), _ptr(accepted_len), _stream(stream)),
            "lsp_view_update")
 
 
-def lsp_prefill(st, b, k, v, h, rows=None, stream=None) -> None:
-    """k, v: [L][t][nkv][d], h: [L][t][H] of request b's whole prefix."""
-    f = lsp_target_feats(_ptr(k), _ptr(v), _ptr(h), int(rows if rows is not None else k.shape[1]))
+def lsp_prefill(st, b, k, v, h, rows=None, stream=None, h_rows=0) -> None:
+    """k, v: [L][t][nkv][d], h: [L][t][H] of request b's whole prefix ([L][1][H], the last
+    row only, with h_rows = 1)."""
+    f = lsp_target_feats(_ptr(k), _ptr(v), _ptr(h), int(rows if rows is not None else k.shape[1]),
+                         int(h_rows))
     _check(_f["lsp_prefill"](st, int(b), ctypes.byref(f), _stream(stream)), "lsp_prefill")
 
 

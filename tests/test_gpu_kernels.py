@@ -121,6 +121,37 @@ def test_view_update_matches_oracle(lsp, s):
         lsp.lsp_state_destroy(st)
 
 
+def test_boundary_row_only_features_match_full_rows(lsp):
+    """h_rows = 1 (each request's boundary row only) gives the same state as the full rows,
+    and h_rows values other than 0, 1 and rows are rejected."""
+    s = VU
+    cfg = lsp.make_config(s)
+    a, b2 = lsp.lsp_state_create(cfg), lsp.lsp_state_create(cfg)
+    try:
+        G = synth.make_weights(s, seed=6)["G"].cuda()
+        lsp.lsp_state_init(a, G)
+        lsp.lsp_state_init(b2, G)
+        for r, acc in enumerate([[5, 1, 17], [16, 3, 0], [2, 40, 9]]):
+            rows = max(acc) + 2
+            k, v, h = synth.make_features(s, rows, seed=300 + r, device="cuda")
+            acc_t = torch.tensor(acc, dtype=torch.int32, device="cuda")
+            # the boundary row of each (request, layer); requests with no new row keep row 0
+            idx = (acc_t.long().clamp(min=1) - 1).view(s.C, 1, 1, 1).expand(s.C, s.L, 1, s.H)
+            h_last = torch.gather(h, 2, idx).contiguous()
+            lsp.lsp_view_update(a, k, v, h, acc_t)
+            lsp.lsp_view_update(b2, k, v, h_last, acc_t, rows=rows, h_rows=1)
+        torch.cuda.synchronize()
+        ea, eb = export_state(lsp, a, s), export_state(lsp, b2, s)
+        for key in ea:
+            assert torch.equal(ea[key], eb[key]), key
+        k, v, h = synth.make_features(s, 4, seed=399, device="cuda")
+        with pytest.raises(lsp.LspError):
+            lsp.lsp_view_update(a, k, v, h, torch.ones(s.C, dtype=torch.int32, device="cuda"), h_rows=2)
+    finally:
+        lsp.lsp_state_destroy(a)
+        lsp.lsp_state_destroy(b2)
+
+
 def test_incremental_fold_equals_one_shot_fold(lsp):
     """Eq. summary-update is exact: chunking a prefix never changes the result (fp32 tolerance)."""
     s = VU
