@@ -625,9 +625,13 @@ int launch_qkv_finalize(const QkvParams& p, int dtype, cudaStream_t s) {
   return e == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
 }
 
+// Key splits per query head.  Measured on one GB300 (A/B): Qwen3-8B (4 heads
+// per KV head) 8 warps (2 splits) beat 16 warps by 8.7 us per round; the large
+// shape (5 heads per KV head) gained 27 us per round with 3 splits (15 warps)
+// over 1 split.
 int attn_ksplit(int B, int W, int nq, int nkv) {
   const int rep = nq / nkv;
-  int ks = rep >= 8 ? 1 : 8 / rep;
+  int ks = rep >= 16 ? 1 : (rep <= 4 ? 8 / rep : 16 / rep);
   while (ks > 1) {
     AttnLayout a = attn_layout(B, W, nq, nkv, ks);
     const size_t scratch = (size_t)rep * (ks - 1) * kMergeRec * sizeof(float);
