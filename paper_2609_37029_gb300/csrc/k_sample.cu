@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(kSampThreads, 2) sample_step_kernel(const Samp
         if (p.dst) *reinterpret_cast<float4*>(p.dst + zoff(tile, k)) = z;
         float sc[4] = {z.x, z.y, z.z, z.w};
         if (sample) {
-          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)step, (uint32_t)b, p.round), key);
+          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)step, (uint32_t)(p.b0 + b), p.round), key);
           sc[0] = sc[0] * inv_temp + gumbel_of(x.x);
           sc[1] = sc[1] * inv_temp + gumbel_of(x.y);
           sc[2] = sc[2] * inv_temp + gumbel_of(x.z);
@@ -422,7 +422,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const int v = (t_begin + lt) * 16 + 4 * q;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(g + 8 * h), p.round), key);
+      const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(p.b0 + g + 8 * h), p.round), key);
       gn[j][h][0] = gumbel_of(x.x);
       gn[j][h][1] = gumbel_of(x.y);
       gn[j][h][2] = gumbel_of(x.z);
@@ -687,7 +687,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         if (p.dst) p.dst[((size_t)c * B + s) * V + v] = z;
         float sc = z;
         if (sample) {
-          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)c, p.round), key);
+          const uint4 x = philox4x32_10(make_uint4((uint32_t)(v >> 2), (uint32_t)s, (uint32_t)(p.b0 + c), p.round), key);
           const uint32_t wd = (v & 3) == 0 ? x.x : (v & 3) == 1 ? x.y : (v & 3) == 2 ? x.z : x.w;
           sc = z * inv_temp + gumbel_of(wd);
         }
@@ -869,8 +869,34 @@ static bool persistent_ok(const SampleParams& p, int dtype) {
   return coop_ok();
 }
 
+// More than kPMaxC requests: the requests' proposal chains are independent,
+// so the one-launch loop runs once per group of up to kPMaxC requests
+// whenever every group fits it (the Philox counter keeps the global request
+// index, so the draws are those of one launch over all requests); the
+// per-step kernel covers all C otherwise.
+static SampleParams request_group(const SampleParams& p, int g0) {
+  SampleParams q = p;
+  q.C = std::min(kPMaxC, p.C - g0);
+  q.src = p.src + (size_t)g0 * p.B * p.V;
+  if (p.dst) q.dst = p.dst + (size_t)g0 * p.B * p.V;
+  q.prev = p.prev + (size_t)g0 * p.prev_stride;
+  q.out_tokens = p.out_tokens + (size_t)g0 * p.B;
+  q.b0 = p.b0 + g0;
+  return q;
+}
+
+static int persistent_groups(const SampleParams& p, int dtype) {
+  if (p.C <= kPMaxC) return persistent_ok(p, dtype) || persistent_f32_ok(p, dtype) ? 1 : 0;
+  for (int g0 = 0; g0 < p.C; g0 += kPMaxC) {
+    const SampleParams q = request_group(p, g0);
+    if (!persistent_ok(q, dtype) && !persistent_f32_ok(q, dtype)) return 0;
+  }
+  return (p.C + kPMaxC - 1) / kPMaxC;
+}
+
 int sample_launches(const SampleParams& p, int dtype) {
-  return persistent_ok(p, dtype) || persistent_f32_ok(p, dtype) ? 1 : p.B + 1;
+  const int groups = persistent_groups(p, dtype);
+  return groups > 0 ? groups : p.B + 1;
 }
 
 int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
@@ -879,9 +905,15 @@ int launch_sample(const SampleParams& p, int dtype, cudaStream_t s) {
   if ((reinterpret_cast<uintptr_t>(p.src) | reinterpret_cast<uintptr_t>(p.dst) |
        reinterpret_cast<uintptr_t>(p.Ec) | reinterpret_cast<uintptr_t>(p.Wc)) & 15)
     return LSP_ERR_ARG;
-  if (persistent_ok(p, dtype))
-    return p.rc == 32 ? launch_persistent<2>(p, s) : launch_persistent<4>(p, s);
-  if (persistent_f32_ok(p, dtype)) return launch_persistent_f32(p, s);
+  if (persistent_groups(p, dtype) > 0) {
+    for (int g0 = 0; g0 < p.C; g0 += kPMaxC) {
+      const SampleParams q = request_group(p, g0);
+      const int rc = persistent_ok(q, dtype) ? (q.rc == 32 ? launch_persistent<2>(q, s) : launch_persistent<4>(q, s))
+                                             : launch_persistent_f32(q, s);
+      if (rc != LSP_OK) return rc;
+    }
+    return LSP_OK;
+  }
 
   if (p.nblk > 32 * kMaxPartialsPerLane) return LSP_ERR_SHAPE;
   const int es = dtype == LSP_DTYPE_BF16 ? 2 : 4;

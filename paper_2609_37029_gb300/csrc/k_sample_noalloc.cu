@@ -82,7 +82,7 @@ extern "C" int lsp_sample_noalloc(const float* base_logits, const int32_t* prev_
   if (sync_off + sync_bytes > kStaticScratchBytes) return LSP_ERR_SHAPE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(scratch + sync_off, 0, sync_bytes, s) != cudaSuccess) return LSP_ERR_CUDA;
-  lsp::SampleParams p;
+  lsp::SampleParams p = {};
   p.src = base_logits;
   p.dst = out_logits;
   p.prev = prev_token;

@@ -423,7 +423,7 @@ static int run_sampler(lsp_state* st, const float* src, float* dst, const int32_
                        int prev_stride, const void* Ec, const void* Wc, const lsp_sample_params* sp,
                        int32_t* out_tokens, cudaStream_t s) {
   const lsp_config& c = st->cfg;
-  SampleParams p;
+  SampleParams p = {};
   p.src = src; p.dst = dst; p.prev = prev; p.prev_stride = prev_stride; p.Ec = Ec; p.Wc = Wc;
   p.out_tokens = out_tokens; p.part_val = st->part_val; p.part_idx = st->part_idx;
   p.sync = st->sample_sync; p.err = st->err;

@@ -229,6 +229,7 @@ struct SampleParams {
   float temperature;
   uint32_t round;
   uint64_t seed;
+  int b0;                 // global index of request 0 of this launch (the Philox counter's request word)
 };
 int sample_blocks(int num_sms);
 size_t sample_sync_bytes(int B);
