@@ -516,11 +516,14 @@ static bool use_three_per_sm(long long ctas, int num_sms, int m_pad, int groups)
 // let three CTAs share an SM.  Two groups for the SwiGLU gate/up projection
 // when its tiles fill at least one wave of one CTA per SM but less than one
 // of two and the token count allows it (Qwen3-8B round, M = 256, 192 tiles:
-// gate/up 368 -> 359 us per round, round 1.243 -> 1.231 ms); one otherwise
-// (every other projection and the LM head measured slower with two or three:
-// more CTAs re-stream each weight tile for the same work).
+// gate/up 368 -> 359 us per round, round 1.243 -> 1.231 ms).  Two groups for
+// every projection above 256 tokens (the large shape, M = 512: round 2600 ->
+// 2485 us), where one group would need a 512-column accumulator, one CTA per
+// SM and two 80 KB stages.  One otherwise (at M = 256 every other projection
+// and the LM head measured slower with two or three: more CTAs re-stream each
+// weight tile for the same work).
 static int token_groups(int M, int mode, int n_tiles, int num_sms) {
-  const int g = mode == EPI_SWIGLU && M >= 128 && n_tiles <= 2 * num_sms && n_tiles >= num_sms ? 2 : 1;
+  const int g = (M > 256 || (mode == EPI_SWIGLU && M >= 128 && n_tiles <= 2 * num_sms && n_tiles >= num_sms)) ? 2 : 1;
   if (g == 1) return 1;
   int bn, ntt;
   token_tiling((M + g - 1) / g, &bn, &ntt);

@@ -38,14 +38,17 @@ def test_gate_up_groups_only_for_an_underfilled_single_wave(lsp, sms, groups):
 
 @pytest.mark.parametrize("N", [12288, 9728, 19456])
 def test_token_groups_cover_every_row_once(lsp, N):
-    """Over every token count, the gate/up plan's groups cover each row once with no
-    empty group; the other projections always take one group."""
+    """Over every token count, the plan's groups cover each row once with no empty
+    group; the other projections take two groups exactly when M > 256 (one 256-token
+    tile per CTA instead of a 512-column accumulator)."""
     for M in range(1, 513):
-        _, g, rows = plan(lsp, M, N, 1024, swiglu=1)
-        assert 1 <= g <= 2 and rows % 16 == 0 and rows <= 512
-        assert g * rows >= M > (g - 1) * rows, (M, g, rows)   # covered, last group not empty
-        assert g == 1 or M >= 16 * g
-        assert plan(lsp, M, N, 1024)[1] == 1
+        for sw in (1, 0):
+            _, g, rows = plan(lsp, M, N, 1024, swiglu=sw)
+            assert 1 <= g <= 2 and rows % 16 == 0 and rows <= 512
+            assert g * rows >= M > (g - 1) * rows, (M, g, rows)   # covered, last group not empty
+            assert g == 1 or M >= 16 * g
+            assert rows <= 256 or M <= 256
+        assert plan(lsp, M, N, 1024)[1] == (2 if M > 256 else 1)
 
 
 def test_bad_arguments(lsp):
