@@ -129,6 +129,27 @@ def test_prefill_equals_incremental_fold_on_gpu(lsp):
             lsp.lsp_state_destroy(st)
 
 
+def test_prefill_with_the_last_hidden_row_only(lsp):
+    """h_rows = 1: h carries only the prefix's last row, the one the boundary reads."""
+    s = PF
+    sts = [lsp.lsp_state_create(lsp.make_config(s)) for _ in range(2)]
+    try:
+        G = synth.make_weights(s, seed=3)["G"].cuda()
+        for st in sts:
+            lsp.lsp_state_init(st, G)
+        k, v, h = synth.make_features(s, 300, seed=77)
+        kb, vb, hb = k[2].contiguous().cuda(), v[2].contiguous().cuda(), h[2].contiguous().cuda()
+        lsp.lsp_prefill(sts[0], 2, kb, vb, hb)
+        lsp.lsp_prefill(sts[1], 2, kb, vb, hb[:, -1:].contiguous(), h_rows=1)
+        torch.cuda.synchronize()
+        ea, eb = export_state(lsp, sts[0], s), export_state(lsp, sts[1], s)
+        for key in ea:
+            assert torch.equal(ea[key], eb[key]), key
+    finally:
+        for st in sts:
+            lsp.lsp_state_destroy(st)
+
+
 @pytest.mark.slow
 def test_prefill_128k_at_qwen3_8b_heads_sampled(lsp):
     """128K rows at the Qwen3-8B head shape (32 q / 8 kv x 128, R = 16), one tapped layer:
