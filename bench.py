@@ -13,7 +13,9 @@ init.  The 3.3 GB of projection weights streamed every round exceed the
 129 MB L2, so no explicit flush is needed between timed rounds.
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 oracle on
-the host cores instead (the baseline of this tier).
+the host cores instead (the reference arm: there is no other implementation
+of the method to run).  `--profile-rounds N` only folds the prefix and runs N
+eager rounds, for a profiler.
 """
 from __future__ import annotations
 
