@@ -351,6 +351,14 @@ __global__ void __launch_bounds__(512)
 // ------------------------------------------------------------ fp32 reference shape
 constexpr int kSimpleChunk = 64;    // window / summary rows staged per round trip
 
+// Lanes per block query in the score loop: the largest power of two with
+// lpq * B <= 32 (1 when B > 16).
+__host__ __device__ inline int simple_lpq(int B) {
+  int lpq = 1;
+  while (lpq * 2 * B <= 32) lpq *= 2;
+  return lpq;
+}
+
 // Rows [j0, j0 + nr) of the context list "count window rows, then summary rows"
 // into shared memory as [nr][d] floats: float4 loads (d % 4 == 0), four in
 // flight per thread before their stores.
@@ -378,7 +386,7 @@ __device__ __forceinline__ void stage_rows(float* dst, const float* win, const f
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p, const int whole) {
   extern __shared__ float ssm[];
   const int d = p.d, B = p.B;
   const int rep = p.nq / p.nkv;
@@ -386,8 +394,11 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
   const long long t = p.t[b];
   const int count = (int)(t < p.W ? t : p.W);
   const int ctx = B + count + p.R;
+  // Query rows padded to d + lpq floats: with d a multiple of 32 the lanes of a
+  // score pass (query qi, dims c + lpq k) then fall in distinct banks.
+  const int lpq = simple_lpq(B), dq = d + lpq;
   float* sq = ssm;
-  float* sk = sq + B * d;
+  float* sk = sq + (B * dq + 3) / 4 * 4;
   float* sv = sk + B * d;
   float* ss = sv + B * d;                 // [B][ctx]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
@@ -400,7 +411,7 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
     const size_t mrow = (size_t)(b * B + i) * ldq;
     const size_t col = kind == 0 ? (size_t)h * d : kind == 1 ? (size_t)(p.nq + g) * d
                                                                 : (size_t)(p.nq + p.nkv + g) * d;
-    (kind == 0 ? sq : kind == 1 ? sk : sv)[i * d + e] = to_f(qkv[mrow + col + e]);
+    (kind == 0 ? sq + i * dq : (kind == 1 ? sk : sv) + i * d)[e] = to_f(qkv[mrow + col + e]);
   }
   __syncthreads();
   const size_t wbase = ((size_t)(b * p.L + p.layer) * p.nkv + g) * p.W * d;
@@ -411,22 +422,70 @@ __global__ void __launch_bounds__(256) attn_simple_kernel(const AttnParams p) {
   const float scale = rsqrtf((float)d);
   float* sc = ss + ((size_t)B * ctx + 3) / 4 * 4;   // [kSimpleChunk][d] staged rows (16-B aligned)
   const int nctx = count + p.R;           // window rows, then summary rows
-  // Lanes split into groups of `lpq` per block query (lpq = the largest power
-  // of two with lpq * B <= 32, queries in passes of 32 / lpq); lane c of a
-  // group covers dims c, c + lpq, ... so a score needs log2(lpq) shuffles.
-  int lpq = 1;
-  while (lpq * 2 * B <= 32) lpq *= 2;
+  // Lanes split into groups of `lpq` per block query (queries in passes of
+  // 32 / lpq); lane c of a group covers dims c, c + lpq, ... so a score needs
+  // log2(lpq) shuffles.
   const int qpp = 32 / lpq, qi = lane / lpq, c = lane % lpq;
   auto score = [&](const float* krow, int j) {   // j: context index of the key
     for (int i0 = 0; i0 < B; i0 += qpp) {
       const int i = i0 + qi;
       float part = 0.f;
       if (i < B)
-        for (int e = c; e < d; e += lpq) part = fmaf(sq[i * d + e], krow[e], part);
+        for (int e = c; e < d; e += lpq) part = fmaf(sq[i * dq + e], krow[e], part);
       for (int o = lpq / 2; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
       if (i < B && c == 0) ss[i * ctx + j] = part * scale;
     }
   };
+  if (whole) {
+    // every window and summary key and value row at once (cp.async, one round
+    // trip for all of them; fp32 rows of d floats, 16-byte chunks)
+    float* sK = sc;
+    float* sV = sc + (size_t)nctx * d;
+    const int d4 = d / 4;
+    for (int idx = tid; idx < nctx * d4; idx += blockDim.x) {
+      const int r = idx / d4, c4 = (idx % d4) * 4;
+      const float* srck = r < count ? reinterpret_cast<const float*>(wk) + (size_t)r * d
+                                    : reinterpret_cast<const float*>(Gh) + (size_t)(r - count) * d;
+      const float* srcv = r < count ? reinterpret_cast<const float*>(wv) + (size_t)r * d : Mh + (size_t)(r - count) * d;
+      cp_async16(sK + (size_t)r * d + c4, srck + c4);
+      cp_async16(sV + (size_t)r * d + c4, srcv + c4);
+    }
+    for (int j = warp; j < B; j += nw) score(sk + j * d, j);
+    cp_async_wait_all();
+    __syncthreads();
+    for (int r = warp; r < nctx; r += nw) score(sK + (size_t)r * d, B + r);
+    __syncthreads();
+    for (int i = warp; i < B; i += nw) {
+      float mx = -INFINITY;
+      for (int j = lane; j < ctx; j += 32) mx = fmaxf(mx, ss[i * ctx + j]);
+      mx = warp_max(mx);
+      float sum = 0.f;
+      for (int j = lane; j < ctx; j += 32) {
+        const float e = expf(ss[i * ctx + j] - mx);
+        ss[i * ctx + j] = e;
+        sum += e;
+      }
+      sum = warp_sum(sum);
+      for (int j = lane; j < ctx; j += 32) ss[i * ctx + j] /= sum;
+    }
+    __syncthreads();
+    T* out = static_cast<T*>(p.out);
+    for (int idx = tid; idx < B * d; idx += blockDim.x) {
+      const int i = idx / d, e = idx % d;
+      const float* pr = ss + (size_t)i * ctx;
+      float a = 0.f, a4[4] = {0.f, 0.f, 0.f, 0.f};   // four independent FMA chains
+      for (int j = 0; j < B; ++j) a = fmaf(pr[j], sv[j * d + e], a);
+      int r = 0;
+      for (; r + 4 <= nctx; r += 4) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a4[u] = fmaf(pr[B + r + u], sV[(size_t)(r + u) * d + e], a4[u]);
+      }
+      for (; r < nctx; ++r) a = fmaf(pr[B + r], sV[(size_t)r * d + e], a);
+      a += (a4[0] + a4[1]) + (a4[2] + a4[3]);
+      out[(size_t)(b * B + i) * p.nq * d + (size_t)h * d + e] = from_f<T>(a);
+    }
+    return;
+  }
   // ---- scores: block keys from shared memory, then the window and summary
   // keys staged kSimpleChunk rows at a time (one coalesced round trip each)
   for (int j = warp; j < B; j += nw) score(sk + j * d, j);
@@ -663,7 +722,12 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
       return LSP_ERR_CUDA;
   } else {
     const int ctx = p.B + p.W + p.R;
-    const size_t smem = (size_t)(3 * p.B * p.d + p.B * ctx + 4 + kSimpleChunk * p.d) * sizeof(float);
+    const size_t fixed = (size_t)(3 * p.B * p.d + p.B * simple_lpq(p.B) + 4 + p.B * ctx + 4) * sizeof(float);
+    // all window and summary rows staged at once when they fit (fp32 and d % 4 == 0
+    // for the 16-byte copies), else kSimpleChunk rows at a time
+    const size_t whole_bytes = fixed + (size_t)2 * (p.W + p.R) * p.d * sizeof(float);
+    const int whole = (dtype == LSP_DTYPE_F32 && p.d % 4 == 0 && whole_bytes <= 227 * 1024) ? 1 : 0;
+    const size_t smem = whole ? whole_bytes : fixed + (size_t)kSimpleChunk * p.d * sizeof(float);
     if (smem > 227 * 1024) return LSP_ERR_SHAPE;
     static bool attr32 = false;
     if (!attr32) {
@@ -671,7 +735,7 @@ int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
                            227 * 1024);
       attr32 = true;
     }
-    if (launch_pdl(attn_simple_kernel<float>, dim3(p.C * p.nq), dim3(256), smem, s, p) != cudaSuccess)
+    if (launch_pdl(attn_simple_kernel<float>, dim3(p.C * p.nq), dim3(256), smem, s, p, whole) != cudaSuccess)
       return LSP_ERR_CUDA;
   }
   return cudaGetLastError() == cudaSuccess ? LSP_OK : LSP_ERR_CUDA;
