@@ -9,6 +9,8 @@
 // The block q and k get the per-head RMSNorm and the rotary embedding here,
 // fused into the load of the q/k/v projection output.
 //
+// The bf16 shapes the tcgen05 kernel serves (k_attn_tc.cu) run there, with the
+// q/k/v finalisation folded in; the kernels below cover the rest.
 // attn_mma_kernel (bf16, d = 128): one CTA per (request, KV head) stages the
 // window once in shared memory for all nq/nkv query heads (HBM traffic = one
 // read of the window and summary); each head gets 8 / (nq/nkv) warps (key
@@ -705,8 +707,9 @@ size_t attn_smem_bytes(int B, int W, int nq, int nkv) {
   return a.bytes;
 }
 
-int launch_attention(const AttnParams& p, int dtype, cudaStream_t s) {
+int launch_attention(const AttnParams& p, int dtype, cudaStream_t s, const AttnTcPlan* tc) {
   if (dtype == LSP_DTYPE_BF16) {
+    if (tc && tc->ok) return launch_attention_tc(p, *tc, s);
     if (p.d != kHD || p.B > 16 || p.R > 16) return LSP_ERR_SHAPE;
     const int ks = attn_ksplit(p.B, p.W, p.nq, p.nkv);
     AttnLayout a = attn_layout(p.B, p.W, p.nq, p.nkv, ks);

@@ -247,7 +247,7 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  griddep_launch();
+  if (!p.late_trigger) griddep_launch();
   const uint32_t tmem_base = *tmem_slot;
 
   int issued = 0;
@@ -294,6 +294,10 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
       load_a(i, smem_u32(smem + (size_t)i * stage_bytes), full_bar(i));
     }
     griddep_wait();                       // activations come from the preceding kernel
+    // A late trigger lets the next kernel start only once every kernel before
+    // this one has completed (it may then read their outputs before its own
+    // wait, as the attention does with the view state).
+    if (p.late_trigger) griddep_launch();
     for (int i = 0; i < pre; ++i)
       load_b(i, smem_u32(smem + (size_t)i * stage_bytes) + stage_a, full_bar(i));
     issued = pre;
@@ -435,6 +439,22 @@ static int make_map(CUtensorMap* m, int dtype, const void* ptr, int K, int rows,
                    2, const_cast<void*>(ptr), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? LSP_OK : LSP_ERR_CUDA;
+}
+
+int tmap_2d_bf16_sw128(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t rows, uint64_t row_bytes,
+                       uint32_t box_inner, uint32_t box_rows) {
+  auto enc = encoder();
+  if (!enc) return LSP_ERR_UNSUPPORTED;
+  if (((uintptr_t)ptr & 15) || (row_bytes % 16) || box_inner * 2 > 128 || box_rows < 1 || box_rows > 256)
+    return LSP_ERR_SHAPE;
+  cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+  cuuint32_t box[2] = {box_inner, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? LSP_OK : LSP_ERR_CUDA;
 }
 

@@ -82,6 +82,7 @@ struct lsp_state {
   size_t sample_sync_bytes = 0;
   int nblk = 0;
   // cached projection plans
+  AttnTcPlan attn_tc = {};
   bool have_plans = false;
   PlanKey key;
   GemmOp fuse, lm;
@@ -413,6 +414,17 @@ static int build_plans(lsp_state* st, const lsp_weights* w, float* out_logits) {
                    c.V)) != LSP_OK)
       return rc;
   }
+  {
+    AttnParams ap = {};
+    ap.qkv = st->qkv; ap.win_k = st->win_k; ap.win_v = st->win_v; ap.G = st->G; ap.m = st->m;
+    ap.C = c.C; ap.B = c.B; ap.L = c.L; ap.nq = c.nq; ap.nkv = c.nkv; ap.d = c.d; ap.W = c.W; ap.R = c.R;
+    st->attn_tc.ok = 0;
+    if (dt == LSP_DTYPE_BF16 && (rc = attn_tc_plan(&st->attn_tc, ap)) != LSP_OK && rc != LSP_ERR_SHAPE)
+      return rc;
+    // the tcgen05 attention reads the view state before its dependency wait:
+    // the q/k/v projection before it triggers only after its own wait
+    for (int j = 0; j < c.D; ++j) st->qkv_op[j].p.late_trigger = st->attn_tc.ok;
+  }
   st->key.w = *w;
   st->key.out_logits = out_logits;
   st->have_plans = true;
@@ -464,18 +476,23 @@ int lsp_draft(lsp_state* st, const int32_t* block_tokens, const lsp_weights* w,
   for (int j = 0; j < c.D; ++j) {
     const lsp_layer_weights& lw = w->layer[j];
     if ((rc = gemm_launch(&st->qkv_op[j], s)) != LSP_OK) return rc;
-    QkvParams qp;
-    qp.part = st->part; qp.splits = st->qkv_op[j].p.splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
-    qp.rope = st->rope; qp.out = st->qkv; qp.M = M; qp.B = c.B; qp.nq = c.nq; qp.nkv = c.nkv; qp.d = c.d;
-    qp.eps = c.rms_eps;
-    if ((rc = launch_qkv_finalize(qp, c.dtype, s)) != LSP_OK) return rc;
+    const bool tc_attn = c.dtype == LSP_DTYPE_BF16 && st->attn_tc.ok;
+    if (!tc_attn) {               // the tcgen05 attention finalises q/k/v itself
+      QkvParams qp = {};
+      qp.part = st->part; qp.splits = st->qkv_op[j].p.splits; qp.q_norm = lw.q_norm; qp.k_norm = lw.k_norm;
+      qp.rope = st->rope; qp.out = st->qkv; qp.M = M; qp.B = c.B; qp.nq = c.nq; qp.nkv = c.nkv; qp.d = c.d;
+      qp.eps = c.rms_eps;
+      if ((rc = launch_qkv_finalize(qp, c.dtype, s)) != LSP_OK) return rc;
+    }
     mark(st, ev++, s);
-    AttnParams ap;
+    AttnParams ap = {};
     ap.qkv = st->qkv;
     ap.win_k = st->win_k; ap.win_v = st->win_v; ap.G = st->G; ap.m = st->m; ap.t = st->t;
     ap.out = st->o; ap.C = c.C; ap.B = c.B; ap.L = c.L; ap.nq = c.nq; ap.nkv = c.nkv; ap.d = c.d;
-    ap.W = c.W; ap.R = c.R; ap.layer = c.layer_map[j]; ap.eps = c.rms_eps;
-    if ((rc = launch_attention(ap, c.dtype, s)) != LSP_OK) return rc;
+    ap.W = c.W; ap.R = c.R; ap.layer = c.layer_map[j]; ap.eps = c.rms_eps; ap.err = st->err;
+    ap.part = st->part; ap.splits = st->qkv_op[j].p.splits; ap.q_norm = lw.q_norm; ap.k_norm = lw.k_norm;
+    ap.rope = st->rope;
+    if ((rc = launch_attention(ap, c.dtype, s, &st->attn_tc)) != LSP_OK) return rc;
     mark(st, ev++, s);
     if ((rc = gemm_launch(&st->o_op[j], s)) != LSP_OK) return rc;
     mark(st, ev++, s);
@@ -567,10 +584,12 @@ int lsp_round_launches(lsp_state* st) {
   const lsp_config& c = st->cfg;
   SampleParams p = {};
   p.C = c.C; p.B = c.B; p.V = c.V; p.rc = c.rc; p.num_sms = st->num_sms; p.sync = st->sample_sync;
-  // view update, fuse, combine; per layer q/k/v GEMM + finalize, attention, o, norm, gate/up, down,
-  // norm; LM head; the sampler
+  // view update, fuse, combine; per layer q/k/v GEMM, finalize (not with the
+  // tcgen05 attention, which finalises q/k/v itself), attention, o, norm,
+  // gate/up, down, norm; LM head; the sampler
   const int fuse = (c.flags & LSP_NO_BOUNDARY) ? 0 : 1;
-  return 2 + fuse + 8 * c.D + 1 + sample_launches(p, c.dtype);
+  const int fin = (c.dtype == LSP_DTYPE_BF16 && attn_tc_supported(c.B, c.W, c.R, c.nq, c.nkv, c.d)) ? 0 : 1;
+  return 2 + fuse + (7 + fin) * c.D + 1 + sample_launches(p, c.dtype);
 }
 
 const char* lsp_stage_name(lsp_state* st, int k) {

@@ -51,6 +51,7 @@ struct GemmParams {
   int tma_out;          // 1: the epilogue stages tiles in shared memory and TMA-stores them
   int out_tok;          // tokens per staged output chunk (16 or 32)
   int tok_groups;       // CTAs per weight tile, each over m_pad consecutive tokens
+  int late_trigger;     // 1: let the next kernel launch only after this one's dependency wait
   void* Y;
   int ldy;
   unsigned* err;
@@ -160,8 +161,33 @@ struct AttnParams {
   void* out;              // [M][nq d]
   int C, B, L, nq, nkv, d, W, R, layer;
   float eps;
+  unsigned* err;          // device error word (a bounded wait that gave up)
+  // tcgen05 kernel only: the q/k/v projection's split partials, finalised
+  // inside the attention (sum in split order, q/k RMSNorm, rotary embedding)
+  const float* part;      // [splits][M][(nq+2nkv)d] fp32
+  int splits;
+  const void* q_norm;     // [d]
+  const void* k_norm;     // [d]
+  const float* rope;      // [C][B][d/2][2]
 };
-int launch_attention(const AttnParams& p, int dtype, cudaStream_t s);
+// Tensor maps of the tcgen05 attention (window K and V, summary keys G),
+// built once per state: ok == 0 where the shape is not served
+// (bf16, d = 128, B <= 16, R <= 16, W <= 256 with W % 16 == 0, nq/nkv <= 8,
+// 16 + W + 16 nq/nkv <= 352).
+struct AttnTcPlan {
+  CUtensorMap wk, wv, g;
+  int wbox;               // window rows per TMA box
+  int ok;
+};
+int attn_tc_plan(AttnTcPlan* pl, const AttnParams& p);
+bool attn_tc_supported(int B, int W, int R, int nq, int nkv, int d);
+// tc: the state's plan (null or !ok: the mma.sync kernel).
+int launch_attention(const AttnParams& p, int dtype, cudaStream_t s, const AttnTcPlan* tc);
+int launch_attention_tc(const AttnParams& p, const AttnTcPlan& pl, cudaStream_t s);
+// 2-D bf16 tensor map, 128-byte swizzle: rows x inner elements (row pitch
+// row_bytes), box (box_inner <= 64, box_rows <= 256).
+int tmap_2d_bf16_sw128(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t rows, uint64_t row_bytes,
+                       uint32_t box_inner, uint32_t box_rows);
 
 // ------------------------------------------------------------------ prefill
 struct PrefillParams {
