@@ -43,7 +43,7 @@ constexpr int kTcCols = 512;      // TMEM columns allocated
 constexpr int kTcThreads = 512;   // four warps per TMEM lane quadrant (column quarters)
 constexpr int kTcMaxKeys = 352;   // S columns stay below kTcOcol; shared memory bound
 constexpr int kTcMaxCh = 6;       // 16-column chunks per warp: ceil(352 / 16 / 4)
-constexpr int kTcMaxItems = 5;    // summary value chunks per thread of warps 2-15 (rep <= 8)
+constexpr int kTcMaxItems = 5;    // summary value chunks per thread of the 480 non-TMA threads (rep <= 8)
 
 struct TcLayout {
   int nk, qstride, dup;
@@ -202,7 +202,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
   } else {
-    const int t0 = tid - 64, nt = kTcThreads - 64;
+    // warps 0 and 2-15: 480 threads, indices 0..479
+    const int t0 = warp == 0 ? lane : tid - 32, nt = kTcThreads - 32;
     // ---- summary values M_h (fp32 -> bf16) as value rows 16 + W + 16 h + r
     //      (rows r >= R zero): every load of this thread issued before its stores
     const float* Mp = p.m + (((size_t)(b * p.L + l) * p.nq + (size_t)g * rep) * R) * kTcD;
