@@ -101,6 +101,14 @@ def _run_rounds(lsp, s, prefixes, reqs=None, chunk=1024, device_gen=False):
             lsp.lsp_draft(st, bt.cuda(), lsp.make_weights(wc), sp, toks, z)
             torch.cuda.synchronize()
             assert lsp.lsp_get_error(st) == (lsp.LSP_OK, 0)
+            # the same round again on the same state gives the same bits (a race
+            # inside a kernel -- e.g. two writers of one staged row -- shows here)
+            toks2 = torch.zeros_like(toks)
+            z2 = torch.zeros_like(z)
+            lsp.lsp_draft(st, bt.cuda(), lsp.make_weights(wc), sp, toks2, z2)
+            torch.cuda.synchronize()
+            assert torch.equal(toks, toks2) and torch.equal(z, z2)
+            del z2
             toks_g = toks.cpu().numpy()
             z_g = z.cpu().double().numpy()
             del z
