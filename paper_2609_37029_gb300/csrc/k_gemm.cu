@@ -369,10 +369,16 @@ __global__ void __launch_bounds__(kGemmThreads, kOcc)
     if (!ok) *s_abort = 1;
     tc_fence_after();
     named_bar(1, kEpilogueThreads);
+    // one thread's snapshot of s_abort (which another role may set at any
+    // time), so that all four warps take the same branch below
+    volatile int* s_stop = s_abort + 1;
+    if (r == 0) *s_stop = *s_abort;
+    named_bar(1, kEpilogueThreads);
+    const bool go = *s_stop == 0;
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
-    if (*s_abort == 0 && p.tma_out) {
+    if (go && p.tma_out) {
       epilogue_tma<T>(p, &to, smem, lane_base, tile, tok0, split, r);
-    } else if (*s_abort == 0) {
+    } else if (go) {
       for (int tt = 0; tt < p.n_tok_tiles; ++tt)
         for (int c0 = 0; c0 < p.bn; c0 += 16) {
           float v[16];

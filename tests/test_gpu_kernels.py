@@ -54,6 +54,8 @@ LINEAR_CASES = [
     (256, 256, 1024, "bf16", 12),
     (256, 2560, 1024, "bf16", 8),    # >= 2 CTAs per SM
     (250, 19456, 512, "bf16", 1),    # ragged M, one split, 152 weight tiles
+    (256, 40000, 512, "bf16", 1),    # >= 2 x SMs tiles, fp32 out: the persistent one-CTA-per-SM form
+    (100, 40000, 256, "bf16", 1),    # the same with a ragged token count (112-token tile)
     (8, 128, 256, "f32", 1),
     (64, 384, 260, "f32", 3),
     (64, 384, 520, "f32", 2),
