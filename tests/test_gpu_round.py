@@ -132,16 +132,22 @@ def test_round_matches_oracle(lsp, name):
     {"R": 0},                                   # ablation: w/o global summary
     {"no_boundary": True},                      # ablation: w/o boundary state
     {"B": 7, "W": 0, "R": 0, "no_boundary": True, "temperature": 1.0},
+    {"nq": 10},                                 # 5 query heads per KV head: one copy of each row
+    {"nq": 10, "B": 7, "R": 5},                 # ... with a short block and partial summary slots
+    {"W": 248},                                 # W % 16 != 0: the mma.sync attention + separate finalize
 ])
 def test_round_variants_match_oracle(lsp, variant):
-    """The paper's B = 7 and the three ablation variants through the same kernels."""
+    """The paper's B = 7, the three ablation variants and other query-head groupings
+    through the same kernels."""
     s = synth.SMALL.with_(**variant)
     _run_round(lsp, s, 3000)
 
 
-def test_round_sampled_and_short_prefix(lsp):
-    """Temperature-1 sampling on the small shape, and a prefix shorter than the window."""
-    s = synth.SMALL.with_(temperature=1.0)
+@pytest.mark.parametrize("nq", [8, 10])
+def test_round_sampled_and_short_prefix(lsp, nq):
+    """Temperature-1 sampling on the small shape, and a prefix shorter than the window
+    (empty window slots in the attention), with 4 and 5 query heads per KV head."""
+    s = synth.SMALL.with_(temperature=1.0, nq=nq)
     _run_round(lsp, s, 100)
 
 
