@@ -34,11 +34,7 @@
  *     caller synchronises; calls on different states, and lsp_linear calls
  *     with different workspaces, may overlap from any threads and streams.
  *     The one process-wide buffer is lsp_sample_noalloc's scratch (below).
- *   - Environment variables, read when a kernel is launched, change how the
- *     work is laid out and never what it computes beyond the order of fp32
- *     summation: LSP_PREFILL_CHUNK (prefill K/V stage rows: 16, 32 or 64);
- *     LSP_VIEW_FMA=1 (the FMA view-update kernel instead of the tensor-core
- *     one).  Unset is the measured default.
+ *   - No environment variable changes what the library computes or how.
  */
 #ifndef LSP_H
 #define LSP_H

@@ -293,17 +293,12 @@ int launch_prefill(const PrefillParams& p, int dtype, cudaStream_t s) {
   int seg_rows = (p.rows + kPrefillMaxSeg - 1) / kPrefillMaxSeg;
   seg_rows = std::max(kPfChunk, (seg_rows + kPfChunk - 1) / kPfChunk * kPfChunk);
   const int nseg = (p.rows + seg_rows - 1) / seg_rows;
-  // K/V rows per pipeline stage (LSP_PREFILL_CHUNK=16|32|64 overrides, for measurement)
-  int ch = kPrefillStage;
-  if (const char* v = std::getenv("LSP_PREFILL_CHUNK")) {
-    const int w = std::atoi(v);
-    ch = w == 16 ? 16 : (w == 64 ? 64 : 32);
-  }
+  // K/V rows per pipeline stage
+  constexpr int ch = kPrefillStage;
   const size_t smem = ((size_t)rep * 16 + 4 * ch) * kPfLd * sizeof(bf16);
   if (smem > 227 * 1024) return LSP_ERR_SHAPE;
-  auto kern = ch == 16 ? prefill_partial_kernel<16> : ch == 32 ? prefill_partial_kernel<32> : prefill_partial_kernel<64>;
-  static size_t attr_by[3] = {0, 0, 0};
-  size_t& attr = attr_by[ch == 16 ? 0 : ch == 32 ? 1 : 2];
+  auto kern = prefill_partial_kernel<ch>;
+  static size_t attr = 0;
   if (smem > attr) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return LSP_ERR_CUDA;

@@ -477,9 +477,6 @@ __global__ void __launch_bounds__(MT * 32, vu_min_blocks(MT)) view_update_mma_ke
   }
 }
 
-// LSP_VIEW_FMA=1 keeps the FMA kernel (for measurement)
-static bool view_mma_enabled() { return std::getenv("LSP_VIEW_FMA") == nullptr; }
-
 template <int MT>
 static int launch_mma(const ViewParams& p, cudaStream_t s) {
   const size_t smem = vu_smem_bytes(MT);
@@ -517,7 +514,7 @@ static int launch_dpl(const ViewParams& p, cudaStream_t s) {
 int launch_view_update(const ViewParams& p, int dtype, cudaStream_t s) {
   // tensor-core path: bf16, d = 128, Q = rep * R a multiple of 16 up to 128
   const int Q = (p.nq / p.nkv) * p.R;
-  if (dtype == LSP_DTYPE_BF16 && p.d == 128 && view_mma_enabled() && Q % 16 == 0) {
+  if (dtype == LSP_DTYPE_BF16 && p.d == 128 && Q % 16 == 0) {
     switch (Q / 16) {
       case 1: return launch_mma<1>(p, s);
       case 2: return launch_mma<2>(p, s);
