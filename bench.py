@@ -622,6 +622,13 @@ def round_roofline(s, ms, mean_delta, hbm, tf_burst):
             "roofline_us": t_roof * 1e6, "frac": t_roof * 1e3 / ms}
 
 
+STAGES_NOTE = ("per-stage device time summed over the round's launches, from event records "
+               "between stages (each ends the programmatic overlap at its boundary, so the stages "
+               "sum to more than the round); 'qkv' is the q/k/v projection and 'attention' the "
+               "tcgen05 attention with the q/k/v split sum, q/k norms and rotary folded in (shapes it "
+               "does not serve run a separate finalize kernel inside 'qkv')")
+
+
 def stage_dict(names, st_ms):
     stages = {}
     for n, t in zip(names, st_ms):
@@ -790,6 +797,7 @@ def run_ours(args, dist):
            "config": workload_config(s, prefix),
            "roofline": roofline, "round_roofline": round_roof,
            "stages_us": stage_dict(names, st_ms),
+           "stages_note": STAGES_NOTE,
            "e2e": {"value": job_throughput(dist.world, s.C, s.B, e2e_ms), "unit": UNIT,
                    "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
            "gpu_launches": lsp.lsp_round_launches(st) * args.steps,
